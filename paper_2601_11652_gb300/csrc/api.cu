@@ -1,0 +1,327 @@
+// api.cu -- host side of the C ABI (include/wisp_verify.h): argument checks, workspace
+// carving and kernel launches.  No allocation, no synchronisation on these paths.
+#include <cmath>
+#include <cstring>
+#include <mutex>
+
+#include "accept.cuh"
+#include "attn.cuh"
+
+using namespace wisp;
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceInfo {
+  int sms = 0;
+  bool attrs_done = false;
+};
+DeviceInfo g_dev[kMaxDevices];
+std::mutex g_mu;
+
+Exp2Table make_exp2_table() {
+  Exp2Table t;
+  for (int j = 0; j < 256; ++j) {
+    const double v = std::exp2(j / 256.0);
+    t.hi[j] = (float)v;
+    t.lo[j] = (float)(v - (double)t.hi[j]);
+  }
+  return t;
+}
+const Exp2Table g_exp2 = make_exp2_table();
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+wisp_status device_setup(int *dev_out, int *sms_out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return WISP_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(g_mu);
+  DeviceInfo &d = g_dev[dev];
+  if (!d.attrs_done) {
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return WISP_ERR_CUDA;
+    cudaError_t e = attn_simt_setup();
+    if (e == cudaSuccess) e = accept_setup();
+    if (e != cudaSuccess) return WISP_ERR_CUDA;
+    d.sms = sms;
+    d.attrs_done = true;
+  }
+  *dev_out = dev;
+  *sms_out = d.sms;
+  return WISP_OK;
+}
+
+bool aligned16(const void *p) { return ((uintptr_t)p & 15) == 0; }
+
+wisp_status check_attn(const wisp_attn_args *a) {
+  if (!a) return WISP_ERR_INVALID_ARG;
+  if (a->B < 0 || a->Hq <= 0 || a->Hkv <= 0 || a->Hq % a->Hkv != 0) return WISP_ERR_INVALID_ARG;
+  if (a->D != 64 && a->D != 128) return WISP_ERR_UNSUPPORTED;
+  if (a->block_size != 16) return WISP_ERR_UNSUPPORTED;
+  if (a->qkv_dtype != WISP_F32 && a->qkv_dtype != WISP_BF16) return WISP_ERR_INVALID_ARG;
+  if (a->B == 0) return WISP_OK;
+  if (a->max_blocks_per_seq <= 0 || a->num_blocks <= 0 || a->total_q_rows < a->B) return WISP_ERR_INVALID_ARG;
+  if (!a->draft_lens || !a->context_lens || !a->block_tables || !a->q || !a->k_cache || !a->v_cache || !a->out)
+    return WISP_ERR_INVALID_ARG;
+  if (!aligned16(a->q) || !aligned16(a->k_cache) || !aligned16(a->v_cache) || !aligned16(a->out))
+    return WISP_ERR_INVALID_ARG;
+  if ((int64_t)a->max_blocks_per_seq * a->block_size > INT32_MAX / 2) return WISP_ERR_UNSUPPORTED;
+  return WISP_OK;
+}
+
+int accept_tiles(const wisp_accept_args *c) {
+  const int E = c->logits_dtype == WISP_BF16 ? 8 : 4;
+  return (c->V + 32 * E - 1) / (32 * E);
+}
+
+wisp_status check_accept(const wisp_accept_args *c) {
+  if (!c) return WISP_ERR_INVALID_ARG;
+  if (c->B < 0 || c->V <= 0 || c->total_draft < 0) return WISP_ERR_INVALID_ARG;
+  if (c->logits_dtype != WISP_F32 && c->logits_dtype != WISP_BF16) return WISP_ERR_INVALID_ARG;
+  if (c->B == 0) return WISP_OK;
+  if (c->total_q_rows < c->B) return WISP_ERR_INVALID_ARG;
+  if (!c->draft_lens || !c->target_logits || !c->sample_uniforms || !c->accepted_len || !c->next_token)
+    return WISP_ERR_INVALID_ARG;
+  if (c->total_draft > 0 && (!c->draft_tokens || !c->draft_probs || !c->accept_uniforms))
+    return WISP_ERR_INVALID_ARG;
+  if (accept_tiles(c) > kMaxAcceptCluster * kLargeTilesPerCta) return WISP_ERR_UNSUPPORTED;
+  if ((int64_t)c->B * 8 > INT32_MAX) return WISP_ERR_UNSUPPORTED;
+  return WISP_OK;
+}
+
+Layout make_layout(const wisp_attn_args *a, const wisp_accept_args *c, int sms) {
+  Layout L;
+  const int B = a ? a->B : (c ? c->B : 0);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align256(off + bytes);
+    return at;
+  };
+  L.status = take(sizeof(DeviceStatus));
+  L.q_row_start = take(sizeof(int32_t) * (size_t)(B + 1));
+  L.draft_start = take(sizeof(int32_t) * (size_t)(B + 1));
+  L.req_flag = take(sizeof(int32_t) * (size_t)B);
+  L.plan_header = take(sizeof(PlanHeader));
+  if (a) {
+    L.target_items = sms * kItemsPerSM;
+    L.max_items = (int64_t)L.target_items + (int64_t)B * a->Hkv;
+    L.partial_cap = (int64_t)2 * L.target_items * kMaxRowsPerHead * (a->D + 2);
+    L.req_item_begin = take(sizeof(int32_t) * (size_t)B);
+    L.req_chunks = take(sizeof(int32_t) * (size_t)B);
+    L.items = take(sizeof(WorkItem) * (size_t)L.max_items);
+    L.partials = take(sizeof(float) * (size_t)L.partial_cap);
+  }
+  L.total = off;
+  return L;
+}
+
+template <typename T>
+T *at(void *ws, size_t off) {
+  return reinterpret_cast<T *>(static_cast<char *>(ws) + off);
+}
+
+wisp_status check_ws(void *ws, size_t bytes, const Layout &L) {
+  if (!ws || ((uintptr_t)ws & 255) != 0 || bytes < L.total) return WISP_ERR_WORKSPACE;
+  return WISP_OK;
+}
+
+PlanParams plan_params(const wisp_attn_args *a, const wisp_accept_args *c, void *ws, const Layout &L) {
+  PlanParams pp;
+  std::memset(&pp, 0, sizeof pp);
+  pp.B = a ? a->B : c->B;
+  pp.draft_lens = a ? a->draft_lens : c->draft_lens;
+  pp.request_ids = a ? a->request_ids : c->request_ids;
+  pp.total_q_rows = a ? a->total_q_rows : c->total_q_rows;
+  pp.total_draft = c ? c->total_draft : INT32_MAX;
+  pp.status = at<DeviceStatus>(ws, L.status);
+  pp.q_row_start = at<int32_t>(ws, L.q_row_start);
+  pp.draft_start = at<int32_t>(ws, L.draft_start);
+  pp.req_flag = at<int32_t>(ws, L.req_flag);
+  pp.header = at<PlanHeader>(ws, L.plan_header);
+  if (a) {
+    pp.Hq = a->Hq;
+    pp.Hkv = a->Hkv;
+    pp.D = a->D;
+    pp.max_blocks_per_seq = a->max_blocks_per_seq;
+    pp.block_size = a->block_size;
+    pp.context_lens = a->context_lens;
+    pp.with_attention = 1;
+    pp.target_items = L.target_items;
+    pp.max_items = L.max_items;
+    pp.partial_cap = L.partial_cap;
+    pp.req_item_begin = at<int32_t>(ws, L.req_item_begin);
+    pp.req_chunks = at<int32_t>(ws, L.req_chunks);
+    pp.items = at<WorkItem>(ws, L.items);
+  } else {
+    pp.Hq = pp.Hkv = 1;
+  }
+  return pp;
+}
+
+wisp_status launch_attention(const wisp_attn_args *a, void *ws, const Layout &L, cudaStream_t s) {
+  AttnParams ap;
+  ap.B = a->B;
+  ap.Hq = a->Hq;
+  ap.Hkv = a->Hkv;
+  ap.D = a->D;
+  ap.max_blocks_per_seq = a->max_blocks_per_seq;
+  ap.num_blocks = a->num_blocks;
+  ap.request_ids = a->request_ids;
+  ap.block_tables = a->block_tables;
+  ap.q = a->q;
+  ap.k_cache = a->k_cache;
+  ap.v_cache = a->v_cache;
+  ap.out = a->out;
+  ap.status = at<DeviceStatus>(ws, L.status);
+  ap.req_flag = at<int32_t>(ws, L.req_flag);
+  ap.req_item_begin = at<int32_t>(ws, L.req_item_begin);
+  ap.req_chunks = at<int32_t>(ws, L.req_chunks);
+  ap.header = at<PlanHeader>(ws, L.plan_header);
+  ap.items = at<WorkItem>(ws, L.items);
+  ap.partials = at<float>(ws, L.partials);
+  const bool bf = a->qkv_dtype == WISP_BF16;
+  if (attn_simt_launch(ap, bf, (int)L.max_items, s) != cudaSuccess) return WISP_ERR_CUDA;
+  return attn_combine_launch(ap, bf, s) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
+}
+
+wisp_status launch_accept(const wisp_accept_args *c, void *ws, const Layout &L, cudaStream_t s) {
+  AcceptParams ap;
+  std::memset(&ap, 0, sizeof ap);
+  ap.B = c->B;
+  ap.V = c->V;
+  const bool bf = c->logits_dtype == WISP_BF16;
+  const size_t esz = bf ? 2 : 4;
+  ap.vec_z = ((uintptr_t)c->target_logits % 16 == 0) && ((size_t)c->V * esz % 16 == 0);
+  ap.vec_q = c->draft_probs && ((uintptr_t)c->draft_probs % 16 == 0) && ((size_t)c->V * 4 % 16 == 0);
+  ap.request_ids = c->request_ids;
+  ap.draft_lens = c->draft_lens;
+  ap.logits = c->target_logits;
+  ap.draft_tokens = c->draft_tokens;
+  ap.draft_probs = c->draft_probs;
+  ap.accept_u = c->accept_uniforms;
+  ap.sample_u = c->sample_uniforms;
+  ap.accepted_len = c->accepted_len;
+  ap.next_token = c->next_token;
+  ap.q_row_start = at<int32_t>(ws, L.q_row_start);
+  ap.draft_start = at<int32_t>(ws, L.draft_start);
+  ap.req_flag = at<int32_t>(ws, L.req_flag);
+  ap.status = at<DeviceStatus>(ws, L.status);
+  ap.tab = g_exp2;
+  const int tiles = accept_tiles(c);
+  bool large = false;
+  if (tiles <= kSmallTiles) {
+    ap.cluster = 1;
+  } else {
+    // about 16 tiles (one per warp) per CTA, at most kMaxAcceptCluster CTAs
+    int C = (tiles + 15) / 16;
+    const int need = (tiles + kLargeTilesPerCta - 1) / kLargeTilesPerCta;
+    C = C < need ? need : C;
+    ap.cluster = C > kMaxAcceptCluster ? kMaxAcceptCluster : C;
+    large = true;
+  }
+  const cudaError_t e = accept_launch(ap, bf, large, s);
+  return e == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
+}
+
+wisp_status launch_plan(const wisp_attn_args *a, const wisp_accept_args *c, void *ws, const Layout &L,
+                        cudaStream_t s) {
+  if (cudaMemsetAsync(at<DeviceStatus>(ws, L.status), 0, sizeof(DeviceStatus), s) != cudaSuccess)
+    return WISP_ERR_CUDA;
+  const PlanParams pp = plan_params(a, c, ws, L);
+  plan_kernel<<<1, 1024, 0, s>>>(pp);
+  return cudaGetLastError() == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t wisp_verify_workspace_size(const wisp_attn_args *attn, const wisp_accept_args *acc) {
+  if (!attn && !acc) return 0;
+  if (attn && check_attn(attn) != WISP_OK) return 0;
+  if (acc && check_accept(acc) != WISP_OK) return 0;
+  if (attn && acc && attn->B != acc->B) return 0;
+  int dev = 0, sms = 0;
+  if (device_setup(&dev, &sms) != WISP_OK) return 0;
+  return make_layout(attn, acc, sms).total;
+}
+
+wisp_status wisp_verify_attention(const wisp_attn_args *attn, void *ws, size_t ws_bytes, void *stream) {
+  wisp_status st = check_attn(attn);
+  if (st != WISP_OK) return st;
+  int dev = 0, sms = 0;
+  if ((st = device_setup(&dev, &sms)) != WISP_OK) return st;
+  const Layout L = make_layout(attn, nullptr, sms);
+  if ((st = check_ws(ws, ws_bytes, L)) != WISP_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((st = launch_plan(attn, nullptr, ws, L, s)) != WISP_OK) return st;
+  if (attn->B == 0) return WISP_OK;
+  return launch_attention(attn, ws, L, s);
+}
+
+wisp_status wisp_verify_accept(const wisp_accept_args *acc, void *ws, size_t ws_bytes, void *stream) {
+  wisp_status st = check_accept(acc);
+  if (st != WISP_OK) return st;
+  int dev = 0, sms = 0;
+  if ((st = device_setup(&dev, &sms)) != WISP_OK) return st;
+  const Layout L = make_layout(nullptr, acc, sms);
+  if ((st = check_ws(ws, ws_bytes, L)) != WISP_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((st = launch_plan(nullptr, acc, ws, L, s)) != WISP_OK) return st;
+  if (acc->B == 0) return WISP_OK;
+  return launch_accept(acc, ws, L, s);
+}
+
+wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args *acc, void *ws, size_t ws_bytes,
+                             void *stream) {
+  wisp_status st = check_attn(attn);
+  if (st != WISP_OK) return st;
+  if ((st = check_accept(acc)) != WISP_OK) return st;
+  if (attn->B != acc->B || attn->total_q_rows != acc->total_q_rows) return WISP_ERR_INVALID_ARG;
+  int dev = 0, sms = 0;
+  if ((st = device_setup(&dev, &sms)) != WISP_OK) return st;
+  const Layout L = make_layout(attn, acc, sms);
+  if ((st = check_ws(ws, ws_bytes, L)) != WISP_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((st = launch_plan(attn, acc, ws, L, s)) != WISP_OK) return st;
+  if (attn->B == 0) return WISP_OK;
+  if ((st = launch_attention(attn, ws, L, s)) != WISP_OK) return st;
+  return launch_accept(acc, ws, L, s);
+}
+
+wisp_status wisp_verify_get_device_status(const void *ws, int32_t *code, int64_t *request_id) {
+  if (!ws || !code || !request_id) return WISP_ERR_INVALID_ARG;
+  DeviceStatus h;
+  if (cudaMemcpy(&h, ws, sizeof h, cudaMemcpyDeviceToHost) != cudaSuccess) return WISP_ERR_CUDA;
+  *code = h.code;
+  *request_id = h.code ? h.request_id : -1;
+  return WISP_OK;
+}
+
+const char *wisp_verify_status_string(wisp_status s) {
+  switch (s) {
+    case WISP_OK: return "ok";
+    case WISP_ERR_INVALID_ARG: return "invalid argument";
+    case WISP_ERR_UNSUPPORTED: return "unsupported configuration";
+    case WISP_ERR_CUDA: return "CUDA runtime error";
+    case WISP_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+  }
+  return "unknown status";
+}
+
+const char *wisp_verify_device_code_string(int32_t code) {
+  switch (code) {
+    case WISP_DEV_OK: return "ok";
+    case WISP_DEV_BAD_LENGTH: return "bad length";
+    case WISP_DEV_BAD_BLOCK: return "block id out of range";
+    case WISP_DEV_BAD_TOKEN: return "draft token out of range";
+    case WISP_DEV_BAD_PROB: return "bad probability or logit row";
+    case WISP_DEV_UNSUPPORTED: return "unsupported request shape";
+    case WISP_DEV_TIMEOUT: return "device wait timed out";
+  }
+  return "unknown device code";
+}
+
+}  // extern "C"

@@ -1,0 +1,26 @@
+// attn.cuh -- parameters of the attention kernels.
+#pragma once
+
+#include "plan.cuh"
+
+namespace wisp {
+
+struct AttnParams {
+  int B, Hq, Hkv, D, max_blocks_per_seq, num_blocks;
+  const int64_t *request_ids;
+  const int32_t *block_tables;
+  const void *q, *k_cache, *v_cache;
+  void *out;
+  DeviceStatus *status;
+  const int32_t *req_flag, *req_item_begin, *req_chunks;
+  const PlanHeader *header;
+  const WorkItem *items;
+  float *partials;
+};
+
+// Host launchers (defined next to their kernels).
+cudaError_t attn_simt_setup();  // once per device: shared-memory attributes
+cudaError_t attn_simt_launch(const AttnParams &p, bool bf16, int grid, cudaStream_t s);
+cudaError_t attn_combine_launch(const AttnParams &p, bool bf16, cudaStream_t s);
+
+}  // namespace wisp

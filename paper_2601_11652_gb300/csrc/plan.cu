@@ -1,0 +1,160 @@
+// plan.cu -- one-CTA planner: request offsets, length validation and the split-KV work list.
+//
+// The verification batch (Sec. 4.5) is ragged: request r contributes k_r + 1 query
+// rows and c_r + k_r + 1 keys (L_total = L_cached + L_new, Sec. 4.4).  Lengths
+// live on the device, so the planner runs there: it prefix-sums the row offsets,
+// flags invalid requests, and cuts every (request, KV head) sequence into chunks
+// of at most `chunk_len` keys so that the attention grid has about
+// kItemsPerSM items per SM whatever the length mix.
+#include "plan.cuh"
+
+namespace wisp {
+
+namespace {
+
+constexpr int kThreads = 1024;
+
+__device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
+__device__ __forceinline__ int64_t max64(int64_t a, int64_t b) { return a > b ? a : b; }
+
+// Inclusive block scan of one int64 per thread; returns the inclusive value, *total the block sum.
+__device__ int64_t block_scan(int64_t v, int64_t *s_warp, int64_t *total) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  for (int d = 1; d < 32; d <<= 1) {
+    int64_t o = __shfl_up_sync(0xffffffffu, v, d);
+    if (lane >= d) v += o;
+  }
+  if (lane == 31) s_warp[w] = v;
+  __syncthreads();
+  if (w == 0) {
+    int64_t t = s_warp[lane];
+    for (int d = 1; d < 32; d <<= 1) {
+      int64_t o = __shfl_up_sync(0xffffffffu, t, d);
+      if (lane >= d) t += o;
+    }
+    s_warp[lane] = t;
+  }
+  __syncthreads();
+  int64_t res = v + (w > 0 ? s_warp[w - 1] : 0);
+  *total = s_warp[31];
+  __syncthreads();
+  return res;
+}
+
+}  // namespace
+
+__global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
+  __shared__ int64_t s_warp[32];
+  const int tid = threadIdx.x;
+  const int g = p.Hq > 0 && p.Hkv > 0 ? p.Hq / p.Hkv : 1;
+  const int64_t cap_tokens = (int64_t)p.max_blocks_per_seq * p.block_size;
+
+  // pass 1: offsets (negative lengths count as 0) and validation
+  int64_t carry_q = 0, carry_d = 0, carry_n = 0;
+  for (int base = 0; base < p.B; base += kThreads) {
+    const int r = base + tid;
+    int64_t k = 0, n = 0;
+    int bad = 0;
+    if (r < p.B) {
+      k = p.draft_lens[r];
+      if (k < 0) { bad = WISP_DEV_BAD_LENGTH; k = 0; }
+      if (!bad && k > kMaxDraft) bad = WISP_DEV_UNSUPPORTED;
+      if (p.with_attention) {
+        const int64_t c = p.context_lens[r];
+        if (!bad && (c < 0 || c + k + 1 > cap_tokens)) bad = WISP_DEV_BAD_LENGTH;
+        if (!bad && (int64_t)g * (k + 1) > kMaxRowsPerHead) bad = WISP_DEV_UNSUPPORTED;
+        n = bad ? 0 : c + k + 1;
+      }
+    }
+    int64_t tq, td, tn;
+    const int64_t iq = block_scan(r < p.B ? k + 1 : 0, s_warp, &tq);
+    const int64_t id = block_scan(r < p.B ? k : 0, s_warp, &td);
+    const int64_t in = block_scan(n, s_warp, &tn);
+    (void)in;
+    if (r < p.B) {
+      const int64_t q0 = carry_q + iq - (k + 1), d0 = carry_d + id - k;
+      // a request whose rows fall outside the caller's buffers is never touched
+      if (!bad && (q0 + k + 1 > p.total_q_rows || d0 + k > p.total_draft)) bad = WISP_DEV_BAD_LENGTH;
+      p.q_row_start[r] = (int32_t)min64(q0, INT32_MAX);
+      p.draft_start[r] = (int32_t)min64(d0, INT32_MAX);
+      p.req_flag[r] = bad ? REQ_BAD : REQ_OK;
+      if (bad) report(p.status, bad, p.request_ids, r);
+    }
+    carry_q += tq;
+    carry_d += td;
+    carry_n += tn;
+  }
+  if (tid == 0) {
+    p.q_row_start[p.B] = (int32_t)min64(carry_q, INT32_MAX);
+    p.draft_start[p.B] = (int32_t)min64(carry_d, INT32_MAX);
+    if (carry_q != p.total_q_rows || carry_d != p.total_draft) {
+      // the caller sized its buffers with other totals: flag it (requests that still fit run)
+      atomicCAS(&p.status->code, 0, (int32_t)WISP_DEV_BAD_LENGTH);
+    }
+  }
+  if (!p.with_attention) return;
+  __syncthreads();
+
+  // pass 2: chunk length so that sum over (r, h) of ceil(n_r / chunk_len) is about target_items
+  const int64_t work = carry_n * p.Hkv;
+  int64_t chunk = (work + p.target_items - 1) / max(1, p.target_items);
+  chunk = max64(chunk, kMinChunk);
+  chunk = (chunk + kChunkAlign - 1) / kChunkAlign * kChunkAlign;
+
+  // pass 3: items and partial slots (request-major, then KV head, then chunk)
+  int64_t item_carry = 0, poff_carry = 0;
+  for (int base = 0; base < p.B; base += kThreads) {
+    const int r = base + tid;
+    int64_t n = 0, chunks = 0, rows = 0;
+    if (r < p.B && p.req_flag[r] == REQ_OK) {
+      n = (int64_t)p.context_lens[r] + p.draft_lens[r] + 1;
+      chunks = (n + chunk - 1) / chunk;
+      rows = (int64_t)g * (p.draft_lens[r] + 1);
+    }
+    const int64_t nitems = chunks * p.Hkv;
+    const int64_t pfl = chunks > 1 ? nitems * rows * (p.D + 2) : 0;
+    int64_t ti, tp;
+    const int64_t ii = block_scan(nitems, s_warp, &ti);
+    const int64_t ip = block_scan(pfl, s_warp, &tp);
+    if (r < p.B) {
+      const int64_t first = item_carry + ii - nitems;
+      const int64_t pfirst = poff_carry + ip - pfl;
+      const bool fits = first + nitems <= p.max_items && pfirst + pfl <= p.partial_cap;
+      if (!fits && nitems > 0) {
+        // cannot happen with the host's bounds; refuse the request rather than overflow
+        p.req_flag[r] = REQ_BAD;
+        report(p.status, WISP_DEV_UNSUPPORTED, p.request_ids, r);
+      }
+      p.req_item_begin[r] = (int32_t)first;
+      p.req_chunks[r] = fits ? (int32_t)chunks : 0;
+      if (fits) {
+        for (int64_t h = 0; h < p.Hkv; ++h) {
+          for (int64_t c = 0; c < chunks; ++c) {
+            WorkItem it;
+            it.r = r;
+            it.h = (int32_t)h;
+            it.t0 = (int32_t)(c * chunk);
+            it.t1 = (int32_t)min64(n, (c + 1) * chunk);
+            it.rows = (int32_t)rows;
+            it.poff = chunks > 1 ? (int32_t)(pfirst + (h * chunks + c) * rows * (p.D + 2)) : -1;
+            it.q0 = p.q_row_start[r];
+            it.ctx = p.context_lens[r];
+            p.items[first + h * chunks + c] = it;
+          }
+        }
+      }
+    }
+    item_carry += ti;
+    poff_carry += tp;
+  }
+  if (tid == 0) {
+    PlanHeader hd;
+    hd.n_items = (int32_t)min64(item_carry, p.max_items);
+    hd.chunk_len = (int32_t)chunk;
+    hd.partial_floats = (int32_t)min64(poff_carry, p.partial_cap);
+    for (int i = 0; i < 5; ++i) hd.pad[i] = 0;
+    *p.header = hd;
+  }
+}
+
+}  // namespace wisp

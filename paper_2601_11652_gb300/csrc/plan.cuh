@@ -1,0 +1,62 @@
+// plan.cuh -- workspace layout and the device-side planner shared by the kernels.
+#pragma once
+
+#include "common.cuh"
+
+namespace wisp {
+
+// One unit of attention work: KV tokens [t0, t1) of request r for KV head h.
+struct WorkItem {
+  int32_t r, h, t0, t1;
+  int32_t poff;   // offset (floats) of this item's split partials, -1 if the item covers the whole sequence
+  int32_t rows;   // query rows of the item: (Hq/Hkv) * (k_r + 1)
+  int32_t q0;     // first query row of request r
+  int32_t ctx;    // c_r
+};
+
+struct PlanHeader {
+  int32_t n_items;
+  int32_t chunk_len;
+  int32_t partial_floats;
+  int32_t pad[5];
+};
+
+constexpr int kItemsPerSM = 4;     // target work items per SM for split-KV
+constexpr int kMinChunk = 256;     // never split a sequence below this many tokens
+constexpr int kChunkAlign = 128;   // chunk starts are multiples of the KV tile
+
+// Byte offsets of every region inside the caller's workspace.
+struct Layout {
+  size_t status = 0;          // DeviceStatus (256 B)
+  size_t q_row_start = 0;     // int32 [B+1]
+  size_t draft_start = 0;     // int32 [B+1]
+  size_t req_flag = 0;        // int32 [B]
+  size_t plan_header = 0;     // PlanHeader
+  size_t req_item_begin = 0;  // int32 [B]  first item of request r
+  size_t req_chunks = 0;      // int32 [B]  chunks per KV head of request r
+  size_t items = 0;           // WorkItem [max_items]
+  size_t partials = 0;        // float [partial_cap]
+  size_t total = 0;
+  int64_t max_items = 0;
+  int64_t partial_cap = 0;    // floats
+  int target_items = 0;
+};
+
+struct PlanParams {
+  int B, Hq, Hkv, D, max_blocks_per_seq, block_size;
+  int total_q_rows, total_draft;
+  int with_attention;          // 0: offsets and validation only
+  int target_items;
+  int64_t max_items, partial_cap;
+  const int32_t *draft_lens, *context_lens;
+  const int64_t *request_ids;
+  DeviceStatus *status;
+  int32_t *q_row_start, *draft_start, *req_flag;
+  PlanHeader *header;
+  int32_t *req_item_begin, *req_chunks;
+  WorkItem *items;
+};
+
+__global__ void plan_kernel(const PlanParams p);
+
+}  // namespace wisp
