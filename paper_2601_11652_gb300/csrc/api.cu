@@ -134,7 +134,7 @@ PlanParams plan_params(const wisp_attn_args *a, const wisp_accept_args *c, void 
   pp.draft_lens = a ? a->draft_lens : c->draft_lens;
   pp.request_ids = a ? a->request_ids : c->request_ids;
   pp.total_q_rows = a ? a->total_q_rows : c->total_q_rows;
-  pp.total_draft = c ? c->total_draft : INT32_MAX;
+  pp.total_draft = c ? c->total_draft : -1;
   pp.status = at<DeviceStatus>(ws, L.status);
   pp.q_row_start = at<int32_t>(ws, L.q_row_start);
   pp.draft_start = at<int32_t>(ws, L.draft_start);

@@ -74,7 +74,8 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     if (r < p.B) {
       const int64_t q0 = carry_q + iq - (k + 1), d0 = carry_d + id - k;
       // a request whose rows fall outside the caller's buffers is never touched
-      if (!bad && (q0 + k + 1 > p.total_q_rows || d0 + k > p.total_draft)) bad = WISP_DEV_BAD_LENGTH;
+      if (!bad && (q0 + k + 1 > p.total_q_rows || (p.total_draft >= 0 && d0 + k > p.total_draft)))
+        bad = WISP_DEV_BAD_LENGTH;
       p.q_row_start[r] = (int32_t)min64(q0, INT32_MAX);
       p.draft_start[r] = (int32_t)min64(d0, INT32_MAX);
       p.req_flag[r] = bad ? REQ_BAD : REQ_OK;
@@ -87,7 +88,7 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
   if (tid == 0) {
     p.q_row_start[p.B] = (int32_t)min64(carry_q, INT32_MAX);
     p.draft_start[p.B] = (int32_t)min64(carry_d, INT32_MAX);
-    if (carry_q != p.total_q_rows || carry_d != p.total_draft) {
+    if (carry_q != p.total_q_rows || (p.total_draft >= 0 && carry_d != p.total_draft)) {
       // the caller sized its buffers with other totals: flag it (requests that still fit run)
       atomicCAS(&p.status->code, 0, (int32_t)WISP_DEV_BAD_LENGTH);
     }

@@ -44,7 +44,7 @@ struct Layout {
 
 struct PlanParams {
   int B, Hq, Hkv, D, max_blocks_per_seq, block_size;
-  int total_q_rows, total_draft;
+  int total_q_rows, total_draft;  // total_draft < 0: not checked (attention-only call)
   int with_attention;          // 0: offsets and validation only
   int target_items;
   int64_t max_items, partial_cap;
