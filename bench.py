@@ -1,0 +1,360 @@
+#!/usr/bin/env python
+"""Benchmark of the batched speculative-verification step (WISP, Sec. 4.5).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+One step = one call of wisp_verify_step on one synthetic verification batch:
+paged GQA attention for every request's k+1 new tokens (Sec. 4.4-4.5) and the
+in-order acceptance pass with the extra-token draw (Eq. 1-3).  The default
+workload is the Llama-3-8B-shaped layer with 32 requests (llama3_8b_b32).
+Prints one JSON line (rank 0).  Under torchrun every rank verifies its own
+batch (requests are independent: weak scaling, no collective on the data path).
+
+--impl reference times the fp64 CPU oracle (the baseline this library is
+checked against) on the host cores, on bounded samples of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verified draft tokens/sec per verify step; achieved HBM GB/s (% of GB300 peak)"
+UNIT = "verified_tokens/s"
+FLUSH_BYTES = 512 << 20  # > 4x the 126 MB L2: written between timed steps
+
+
+# --------------------------------------------------------------------------
+# algorithmic bytes (what the method must move; per step)
+# --------------------------------------------------------------------------
+def attention_bytes(b) -> int:
+    s = 2 if b.dtype == "bf16" else 4
+    n = b.context_lens.astype(np.int64) + b.draft_lens + 1
+    kv = int(n.sum()) * b.Hkv * b.D * 2 * s          # K and V of every visible token, read once
+    qo = int(b.total_q_rows) * b.Hq * b.D * 2 * s     # Q read, O written
+    bt = int(((n + 15) // 16).sum()) * 4              # block-table entries
+    return kv + qo + bt
+
+
+def accept_bytes(b, L) -> int:
+    s = 2 if b.dtype == "bf16" else 4
+    L = np.asarray(L, np.int64)
+    k = b.draft_lens.astype(np.int64)
+    rows = int((L + 1).sum()) * b.V * s               # logit rows 0..L (the walk stops at the first rejection)
+    qrow = int((L < k).sum()) * b.V * 4               # the draft row at the rejection (residual draw)
+    decisions = int(np.minimum(L + 1, k).sum())
+    gathers = decisions * (32 + 32 + 4 + 4)           # sectors of z(y), q(y); token, uniform
+    return rows + qrow + gathers + b.B * 16
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def _kernel_sha() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2601_11652_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def _profile_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if it matches this source."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    sha = re.search(r"kernel_source_sha:\s*(\w+)", text)
+    tr = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    if not sha or not tr or sha.group(1) != _kernel_sha():
+        return None
+    return float(tr.group(1))
+
+
+# --------------------------------------------------------------------------
+# clocks during the timed region
+# --------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_bench_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, flags in rows for i, v in enumerate(flags) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------------------------
+# oracle timing (cpu_baseline, and the reference arm)
+# --------------------------------------------------------------------------
+def time_oracle(batch, budget_s: float, start: int = 0):
+    """Run the oracle (attention + acceptance) on consecutive requests until budget_s is spent."""
+    import oracle
+    threads = os.cpu_count() or 1
+    t0 = time.perf_counter()
+    done, verified = 0, 0
+    r = start
+    while True:
+        sub = batch.subset([r % batch.B])
+        oracle.attention(sub, nthreads=threads)
+        res = oracle.accept(sub, nthreads=threads)
+        verified += int(res["accepted_len"].sum())
+        done += 1
+        r += 1
+        if time.perf_counter() - t0 >= budget_s or done >= 4 * batch.B:
+            break
+    return done, verified, time.perf_counter() - t0, threads
+
+
+def cpu_baseline(batch, budget_s=10.0):
+    done, verified, dt, threads = time_oracle(batch, budget_s)
+    return {"value": verified / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"{done} requests of {batch.name} (attention + acceptance, fp64), {dt:.1f} s"}
+
+
+def run_reference(args, batch):
+    """The oracle as the reference arm: each step is a bounded sample of the workload."""
+    t_one = time_oracle(batch, 0.0)[2]
+    per_step = max(1, int(3.0 / max(t_one, 1e-3)))
+    for i in range(args.warmup):
+        time_oracle(batch, 0.0, start=i)
+    ms, verified, done, threads = [], 0, 0, 1
+    for i in range(args.steps):
+        d, v, dt, threads = 0, 0, 0.0, threads
+        t0 = time.perf_counter()
+        for j in range(per_step):
+            dd, vv, _, threads = time_oracle(batch, 0.0, start=i * per_step + j)
+            d += dd
+            v += vv
+        dt = time.perf_counter() - t0
+        ms.append(dt * 1e3)
+        verified += v
+        done += d
+    total_s = sum(ms) / 1e3
+    value = verified / total_s
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": sum(ms) / len(ms),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": _config(batch, args),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                             "sample": f"{per_step} request(s) of {batch.name} per step, {done} in total"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def _config(batch, args):
+    return {"workload": batch.name, "B": batch.B, "Hq": batch.Hq, "Hkv": batch.Hkv, "D": batch.D, "V": batch.V,
+            "kv_tokens": batch.kv_tokens(), "draft_tokens": batch.total_draft, "block_size": 16,
+            "kv_dtype": batch.dtype, "accumulate": "fp32", "parallelism": f"replicas{args.gpus}",
+            "l2": "flushed between timed steps (512 MiB write)"}
+
+
+# --------------------------------------------------------------------------
+# our arm
+# --------------------------------------------------------------------------
+def _time_loop(fn, steps, flush, torch):
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    for i in range(steps):
+        flush.zero_()
+        starts[i].record()
+        fn()
+        ends[i].record()
+    torch.cuda.synchronize()
+    return [s.elapsed_time(e) for s, e in zip(starts, ends)]
+
+
+def run_ours(args, batch, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2601_11652_gb300 import build
+    from paper_2601_11652_gb300.device_batch import DeviceBatch
+
+    build.build()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    db = DeviceBatch.from_host(batch, device=dev)
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    for _ in range(max(3, args.warmup)):
+        flush.zero_()
+        db.step()
+    torch.cuda.synchronize()
+    code, rid = db.device_status()
+    if code != 0:
+        raise RuntimeError(f"device status {code} at request {rid}")
+    res = db.results()
+    L = res["accepted_len"]
+    verified = int(L.sum())
+
+    sampler = ClockSampler(local_rank) if rank == 0 else None
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.start()
+        time.sleep(0.3)
+    ms = _time_loop(db.step, args.steps, flush, torch)
+    clocks = sampler.stop() if sampler else None
+    torch.cuda.synchronize()
+    total_ms = sum(ms)
+    verified_all = verified
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+        v = torch.tensor([verified], device=dev, dtype=torch.int64)
+        dist.all_reduce(v, op=dist.ReduceOp.SUM)
+        verified_all = int(v.item())
+        dist.barrier()
+    ms_per_step = total_ms / args.steps
+    value = verified_all / (ms_per_step / 1e3)
+
+    # per-entry-point timings (separate loops, after the timed region)
+    n_sub = min(args.steps, 50)
+    attn_ms = statistics.mean(_time_loop(db.attention, n_sub, flush, torch))
+    acc_ms = statistics.mean(_time_loop(db.accept, n_sub, flush, torch))
+    ab, cb = attention_bytes(batch), accept_bytes(batch, L)
+    peak, peak_kind = _peaks()
+    attn_gbs = ab / (attn_ms * 1e-3) / 1e9
+    acc_gbs = cb / (acc_ms * 1e-3) / 1e9
+
+    # end to end: per-step inputs from pinned host memory, results back to the host
+    e2e = _e2e(db, batch, args, flush, torch, verified)
+
+    if rank != 0:
+        return
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": batch.dtype, "data": "synthetic", "config": _config(batch, args),
+            "roofline": {"bound": "hbm", "kernel": "attention (plan + split-KV attention + combine)",
+                         "achieved": attn_gbs, "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
+                         "frac": attn_gbs / peak, "traffic": _profile_traffic("attention", batch.name),
+                         "algorithmic_bytes_per_launch": ab},
+            "accept_roofline": {"bound": "hbm", "achieved": acc_gbs, "peak": peak, "unit": "GB/s",
+                                "frac": acc_gbs / peak, "algorithmic_bytes_per_launch": cb,
+                                "traffic": _profile_traffic("accept", batch.name)},
+            "step_algorithmic_gbs": (ab + cb) / (ms_per_step * 1e-3) / 1e9,
+            "emitted_tokens_per_s": (verified_all + batch.B * world) / (ms_per_step / 1e3),
+            "mean_acceptance": float(verified / max(1, batch.total_draft)),
+            "cpu_baseline": cpu_baseline(batch),
+            "e2e": e2e, "gpu_launches": 4 * args.steps, "clocks": clocks}
+    print(json.dumps(line), flush=True)
+
+
+def _e2e(db, batch, args, flush, torch, verified):
+    t = db.t
+    names = ["request_ids", "draft_lens", "context_lens", "block_tables", "q", "logits", "draft_tokens",
+             "draft_probs", "accept_u", "sample_u"]
+    host = {n: torch.empty(t[n].shape, dtype=t[n].dtype, pin_memory=True) for n in names}
+    for n in names:
+        host[n].copy_(t[n].cpu())
+    out_L = torch.empty(batch.B, dtype=torch.int32, pin_memory=True)
+    out_T = torch.empty(batch.B, dtype=torch.int32, pin_memory=True)
+    h2d = sum(host[n].numel() * host[n].element_size() for n in names)
+    d2h = 2 * batch.B * 4
+
+    def one():
+        for n in names:
+            t[n].copy_(host[n], non_blocking=True)
+        db.step()
+        out_L.copy_(t["accepted_len"], non_blocking=True)
+        out_T.copy_(t["next_token"], non_blocking=True)
+
+    for _ in range(3):
+        flush.zero_()
+        one()
+    torch.cuda.synchronize()
+    n = min(args.steps, 50)
+    ms = statistics.mean(_time_loop(one, n, flush, torch))
+    assert int(out_L.sum()) == verified
+    return {"value": verified / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": ms, "steps": n,
+            "note": "the paged KV cache (prefix cache) stays resident in HBM; every other input is copied in"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default="llama3_8b_b32")
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    args = ap.parse_args()
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    local_rank = int(os.environ.get("LOCAL_RANK", 0))
+    from paper_2601_11652_gb300 import workload as wl
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        run_reference(args, wl.make_batch(args.workload))
+        return
+    # each rank verifies its own copy of the batch (independent requests, no collective)
+    batch = wl.make_batch(args.workload)
+    run_ours(args, batch, rank, world, local_rank)
+
+
+if __name__ == "__main__":
+    main()

@@ -42,6 +42,7 @@ wisp_status device_setup(int *dev_out, int *sms_out) {
     int sms = 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return WISP_ERR_CUDA;
     cudaError_t e = attn_simt_setup();
+    if (e == cudaSuccess) e = attn_tc_setup();
     if (e == cudaSuccess) e = accept_setup();
     if (e != cudaSuccess) return WISP_ERR_CUDA;
     d.sms = sms;
@@ -182,7 +183,13 @@ wisp_status launch_attention(const wisp_attn_args *a, void *ws, const Layout &L,
   ap.items = at<WorkItem>(ws, L.items);
   ap.partials = at<float>(ws, L.partials);
   const bool bf = a->qkv_dtype == WISP_BF16;
-  if (attn_simt_launch(ap, bf, (int)L.max_items, s) != cudaSuccess) return WISP_ERR_CUDA;
+  if (bf) {
+    // persistent tensor-core kernel: one CTA per SM
+    const int grid = (int)(L.max_items < L.target_items / kItemsPerSM ? L.max_items : L.target_items / kItemsPerSM);
+    if (attn_tc_launch(ap, grid, s) != cudaSuccess) return WISP_ERR_CUDA;
+  } else {
+    if (attn_simt_launch(ap, bf, (int)L.max_items, s) != cudaSuccess) return WISP_ERR_CUDA;
+  }
   return attn_combine_launch(ap, bf, s) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
 }
 

@@ -22,5 +22,8 @@ struct AttnParams {
 cudaError_t attn_simt_setup();  // once per device: shared-memory attributes
 cudaError_t attn_simt_launch(const AttnParams &p, bool bf16, int grid, cudaStream_t s);
 cudaError_t attn_combine_launch(const AttnParams &p, bool bf16, cudaStream_t s);
+// tcgen05 / TMA kernel for bf16 KV, D in {64, 128}; `grid` persistent CTAs
+cudaError_t attn_tc_setup();
+cudaError_t attn_tc_launch(const AttnParams &p, int grid, cudaStream_t s);
 
 }  // namespace wisp

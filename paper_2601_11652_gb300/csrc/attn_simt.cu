@@ -171,7 +171,8 @@ __global__ void __launch_bounds__(128) attn_combine_kernel(const AttnParams p) {
   if (r >= p.B || p.req_flag[r] != REQ_OK) return;
   const int chunks = p.req_chunks[r];
   if (chunks <= 1) return;
-  const WorkItem first = p.items[p.req_item_begin[r] + h * chunks];
+  const WorkItem *items = p.items + p.req_item_begin[r] + h * chunks;
+  const WorkItem first = items[0];
   const int R = first.rows;
   const int g = p.Hq / p.Hkv;
   T *out = static_cast<T *>(p.out);
@@ -179,12 +180,12 @@ __global__ void __launch_bounds__(128) attn_combine_kernel(const AttnParams p) {
     const int rho = i / D, d = i % D;
     float m = -INFINITY;
     for (int c = 0; c < chunks; ++c) {
-      const float *part = p.partials + first.poff + (int64_t)c * R * (D + 2);
+      const float *part = p.partials + items[c].poff;
       m = fmaxf(m, part[R * D + rho]);
     }
     float num = 0.0f, den = 0.0f;
     for (int c = 0; c < chunks; ++c) {
-      const float *part = p.partials + first.poff + (int64_t)c * R * (D + 2);
+      const float *part = p.partials + items[c].poff;
       const float mc = part[R * D + rho];
       if (mc == -INFINITY) continue;
       const float w = exp2f(mc - m);

@@ -113,7 +113,9 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
       rows = (int64_t)g * (p.draft_lens[r] + 1);
     }
     const int64_t nitems = chunks * p.Hkv;
-    const int64_t pfl = chunks > 1 ? nitems * rows * (p.D + 2) : 0;
+    // each split item's partials start on a 16-byte boundary (vector stores)
+    const int64_t slot = (rows * (p.D + 2) + 3) / 4 * 4;
+    const int64_t pfl = chunks > 1 ? nitems * slot : 0;
     int64_t ti, tp;
     const int64_t ii = block_scan(nitems, s_warp, &ti);
     const int64_t ip = block_scan(pfl, s_warp, &tp);
@@ -137,7 +139,7 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
             it.t0 = (int32_t)(c * chunk);
             it.t1 = (int32_t)min64(n, (c + 1) * chunk);
             it.rows = (int32_t)rows;
-            it.poff = chunks > 1 ? (int32_t)(pfirst + (h * chunks + c) * rows * (p.D + 2)) : -1;
+            it.poff = chunks > 1 ? (int32_t)(pfirst + (h * chunks + c) * slot) : -1;
             it.q0 = p.q_row_start[r];
             it.ctx = p.context_lens[r];
             p.items[first + h * chunks + c] = it;
