@@ -125,6 +125,7 @@ typedef struct {
  * accepted: if L < k_r the extra token is the inverse-CDF draw (ascending token ids, first t
  * whose cumulative mass is strictly greater than u * total) from max(0, p_L - q_{L+1}); if
  * that residual has no mass, or L == k_r, the draw is from p_L.
+ * Supported: 1 <= V <= 2^24.
  * The kernel decides every comparison exactly up to about 1e-13 relative error: it computes
  * the row normaliser in fp32 with a certified error bound and recomputes it in double-float
  * arithmetic whenever a decision lies inside that bound.

@@ -5,10 +5,16 @@
 
 namespace wisp {
 
+constexpr int kAcceptThreads = 256;  // 8 warps per CTA
+constexpr int kMaxAcceptCluster = 8;
+constexpr int kPreload = 256;        // decision inputs gathered up front for the first rows
+
 struct AcceptParams {
   int B, V;
   int cluster;        // CTAs per request (1..8), = cluster size of the launch
+  int vpc;            // 16-byte vectors of a row per CTA (multiple of 32)
   int vec_z, vec_q;   // 1 if logit rows / draft-prob rows are 16-byte aligned for vector loads
+  int prefetch;       // 1: prefetch the next logit row into L2 while deciding the current one
   const int64_t *request_ids;
   const int32_t *draft_lens;
   const void *logits;
@@ -21,13 +27,8 @@ struct AcceptParams {
   Exp2Table tab;
 };
 
-// Kernel shapes: SMALL serves rows of at most kSmallTiles 16-byte tiles with one CTA;
-// LARGE serves up to 8 CTAs per request with kLargeTilesPerCta tiles each.
-constexpr int kSmallTiles = 16;
-constexpr int kLargeTilesPerCta = 256;
-constexpr int kMaxAcceptCluster = 8;
-
 cudaError_t accept_setup();  // once per device: shared-memory attributes
-cudaError_t accept_launch(const AcceptParams &p, bool bf16, bool large, cudaStream_t s);
+// rounds = ceil(vpc / kAcceptThreads): sizes the per-(round, warp) draw partials
+cudaError_t accept_launch(const AcceptParams &p, bool bf16, cudaStream_t s);
 
 }  // namespace wisp

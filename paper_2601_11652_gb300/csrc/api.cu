@@ -86,7 +86,7 @@ wisp_status check_accept(const wisp_accept_args *c) {
     return WISP_ERR_INVALID_ARG;
   if (c->total_draft > 0 && (!c->draft_tokens || !c->draft_probs || !c->accept_uniforms))
     return WISP_ERR_INVALID_ARG;
-  if (accept_tiles(c) > kMaxAcceptCluster * kLargeTilesPerCta) return WISP_ERR_UNSUPPORTED;
+  if (c->V > (1 << 24)) return WISP_ERR_UNSUPPORTED;  // vocabulary limit of the acceptance kernel
   if ((int64_t)c->B * 8 > INT32_MAX) return WISP_ERR_UNSUPPORTED;
   return WISP_OK;
 }
@@ -111,6 +111,7 @@ Layout make_layout(const wisp_attn_args *a, const wisp_accept_args *c, int sms) 
     L.partial_cap = (int64_t)2 * L.target_items * kMaxRowsPerHead * (a->D + 2);
     L.req_item_begin = take(sizeof(int32_t) * (size_t)B);
     L.req_chunks = take(sizeof(int32_t) * (size_t)B);
+    L.pair_done = take(sizeof(int32_t) * (size_t)B * a->Hkv);
     L.items = take(sizeof(WorkItem) * (size_t)L.max_items);
     L.partials = take(sizeof(float) * (size_t)L.partial_cap);
   }
@@ -154,6 +155,7 @@ PlanParams plan_params(const wisp_attn_args *a, const wisp_accept_args *c, void 
     pp.partial_cap = L.partial_cap;
     pp.req_item_begin = at<int32_t>(ws, L.req_item_begin);
     pp.req_chunks = at<int32_t>(ws, L.req_chunks);
+    pp.pair_done = at<int32_t>(ws, L.pair_done);
     pp.items = at<WorkItem>(ws, L.items);
   } else {
     pp.Hq = pp.Hkv = 1;
@@ -180,20 +182,23 @@ wisp_status launch_attention(const wisp_attn_args *a, void *ws, const Layout &L,
   ap.req_item_begin = at<int32_t>(ws, L.req_item_begin);
   ap.req_chunks = at<int32_t>(ws, L.req_chunks);
   ap.header = at<PlanHeader>(ws, L.plan_header);
+  ap.header_mut = at<PlanHeader>(ws, L.plan_header);
   ap.items = at<WorkItem>(ws, L.items);
   ap.partials = at<float>(ws, L.partials);
+  ap.pair_done = at<int32_t>(ws, L.pair_done);
   const bool bf = a->qkv_dtype == WISP_BF16;
   if (bf) {
     // persistent tensor-core kernel: one CTA per SM
     const int grid = (int)(L.max_items < L.target_items / kItemsPerSM ? L.max_items : L.target_items / kItemsPerSM);
-    if (attn_tc_launch(ap, grid, s) != cudaSuccess) return WISP_ERR_CUDA;
-  } else {
-    if (attn_simt_launch(ap, bf, (int)L.max_items, s) != cudaSuccess) return WISP_ERR_CUDA;
+    // the work counter lives in the plan header written by the planner on this stream
+    // split items are merged inside the kernel by the last chunk to finish
+    return attn_tc_launch(ap, grid, s) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
   }
+  if (attn_simt_launch(ap, bf, (int)L.max_items, s) != cudaSuccess) return WISP_ERR_CUDA;
   return attn_combine_launch(ap, bf, s) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
 }
 
-wisp_status launch_accept(const wisp_accept_args *c, void *ws, const Layout &L, cudaStream_t s) {
+wisp_status launch_accept(const wisp_accept_args *c, void *ws, const Layout &L, int sms, cudaStream_t s) {
   AcceptParams ap;
   std::memset(&ap, 0, sizeof ap);
   ap.B = c->B;
@@ -216,19 +221,18 @@ wisp_status launch_accept(const wisp_accept_args *c, void *ws, const Layout &L, 
   ap.req_flag = at<int32_t>(ws, L.req_flag);
   ap.status = at<DeviceStatus>(ws, L.status);
   ap.tab = g_exp2;
-  const int tiles = accept_tiles(c);
-  bool large = false;
-  if (tiles <= kSmallTiles) {
-    ap.cluster = 1;
-  } else {
-    // about 16 tiles (one per warp) per CTA, at most kMaxAcceptCluster CTAs
-    int C = (tiles + 15) / 16;
-    const int need = (tiles + kLargeTilesPerCta - 1) / kLargeTilesPerCta;
-    C = C < need ? need : C;
-    ap.cluster = C > kMaxAcceptCluster ? kMaxAcceptCluster : C;
-    large = true;
-  }
-  const cudaError_t e = accept_launch(ap, bf, large, s);
+  // one cluster of C CTAs per request: enough CTAs to fill the GPU, each owning a slice of
+  // every row in whole warp tiles (32 vectors of 16 bytes)
+  const int E = bf ? 8 : 4;
+  const int64_t nvec = ((int64_t)c->V + E - 1) / E;
+  const int64_t want = ((int64_t)4 * sms + c->B - 1) / c->B;
+  int64_t C = want < 1 ? 1 : (want > kMaxAcceptCluster ? kMaxAcceptCluster : want);
+  const int64_t max_c = (nvec + 31) / 32;
+  if (C > max_c) C = max_c;
+  ap.cluster = (int)C;
+  ap.vpc = (int)(((nvec + C - 1) / C + 31) / 32 * 32);
+  ap.prefetch = c->B < sms ? 1 : 0;
+  const cudaError_t e = accept_launch(ap, bf, s);
   return e == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
 }
 
@@ -278,7 +282,7 @@ wisp_status wisp_verify_accept(const wisp_accept_args *acc, void *ws, size_t ws_
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if ((st = launch_plan(nullptr, acc, ws, L, s)) != WISP_OK) return st;
   if (acc->B == 0) return WISP_OK;
-  return launch_accept(acc, ws, L, s);
+  return launch_accept(acc, ws, L, sms, s);
 }
 
 wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args *acc, void *ws, size_t ws_bytes,
@@ -295,7 +299,7 @@ wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args 
   if ((st = launch_plan(attn, acc, ws, L, s)) != WISP_OK) return st;
   if (attn->B == 0) return WISP_OK;
   if ((st = launch_attention(attn, ws, L, s)) != WISP_OK) return st;
-  return launch_accept(acc, ws, L, s);
+  return launch_accept(acc, ws, L, sms, s);
 }
 
 wisp_status wisp_verify_get_device_status(const void *ws, int32_t *code, int64_t *request_id) {

@@ -14,8 +14,10 @@ struct AttnParams {
   DeviceStatus *status;
   const int32_t *req_flag, *req_item_begin, *req_chunks;
   const PlanHeader *header;
+  PlanHeader *header_mut;  // same object: the work counter
   const WorkItem *items;
   float *partials;
+  int32_t *pair_done;  // [B * Hkv] finished chunks of each split (request, head), zeroed by the planner
 };
 
 // Host launchers (defined next to their kernels).

@@ -164,36 +164,54 @@ static size_t attn_simt_smem_bytes(int R, int D) {
 }
 
 // Merge the split partials of one (request, KV head): O = sum_c acc_c 2^(m_c - m) / sum_c l_c 2^(m_c - m).
+// One warp per query row: the chunk weights are formed once per row, each lane owns D/32
+// consecutive output elements and reads the chunk accumulators as 8- or 16-byte vectors.
 template <typename T, int D>
 __global__ void __launch_bounds__(128) attn_combine_kernel(const AttnParams p) {
+  constexpr int PER = D / 32;  // 2 or 4 floats per lane
   const int pair = blockIdx.x;
   const int r = pair / p.Hkv, h = pair % p.Hkv;
   if (r >= p.B || p.req_flag[r] != REQ_OK) return;
   const int chunks = p.req_chunks[r];
   if (chunks <= 1) return;
   const WorkItem *items = p.items + p.req_item_begin[r] + h * chunks;
-  const WorkItem first = items[0];
-  const int R = first.rows;
+  const int R = items[0].rows;
+  const int q0 = items[0].q0;
   const int g = p.Hq / p.Hkv;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   T *out = static_cast<T *>(p.out);
-  for (int i = threadIdx.x; i < R * D; i += blockDim.x) {
-    const int rho = i / D, d = i % D;
+  for (int rho = warp; rho < R; rho += 4) {
     float m = -INFINITY;
-    for (int c = 0; c < chunks; ++c) {
-      const float *part = p.partials + items[c].poff;
-      m = fmaxf(m, part[R * D + rho]);
-    }
-    float num = 0.0f, den = 0.0f;
+    for (int c = lane; c < chunks; c += 32) m = fmaxf(m, p.partials[items[c].poff + R * D + rho]);
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    float acc[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) acc[i] = 0.0f;
+    float den = 0.0f;
     for (int c = 0; c < chunks; ++c) {
       const float *part = p.partials + items[c].poff;
       const float mc = part[R * D + rho];
       if (mc == -INFINITY) continue;
       const float w = exp2f(mc - m);
-      num = fmaf(part[i], w, num);
       den = fmaf(part[R * D + R + rho], w, den);
+      const float *src = part + (int64_t)rho * D + lane * PER;
+      if (PER == 4) {
+        const float4 v = *reinterpret_cast<const float4 *>(src);
+        acc[0] = fmaf(v.x, w, acc[0]);
+        acc[1] = fmaf(v.y, w, acc[1]);
+        acc[2] = fmaf(v.z, w, acc[2]);
+        acc[3] = fmaf(v.w, w, acc[3]);
+      } else {
+        const float2 v = *reinterpret_cast<const float2 *>(src);
+        acc[0] = fmaf(v.x, w, acc[0]);
+        acc[1] = fmaf(v.y, w, acc[1]);
+      }
     }
+    const float inv = 1.0f / den;
     const int j = rho / g, hh = rho % g;
-    st<T>(out, ((int64_t)(first.q0 + j) * p.Hq + h * g + hh) * D + d, num / den);
+    const int64_t o0 = ((int64_t)(q0 + j) * p.Hq + h * g + hh) * D + lane * PER;
+#pragma unroll
+    for (int i = 0; i < PER; ++i) st<T>(out, o0 + i, acc[i] * inv);
   }
 }
 

@@ -129,6 +129,7 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
         report(p.status, WISP_DEV_UNSUPPORTED, p.request_ids, r);
       }
       p.req_item_begin[r] = (int32_t)first;
+      for (int h = 0; h < p.Hkv; ++h) p.pair_done[(int64_t)r * p.Hkv + h] = 0;
       p.req_chunks[r] = fits ? (int32_t)chunks : 0;
       if (fits) {
         for (int64_t h = 0; h < p.Hkv; ++h) {
@@ -155,7 +156,8 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     hd.n_items = (int32_t)min64(item_carry, p.max_items);
     hd.chunk_len = (int32_t)chunk;
     hd.partial_floats = (int32_t)min64(poff_carry, p.partial_cap);
-    for (int i = 0; i < 5; ++i) hd.pad[i] = 0;
+    hd.next_item = 0;
+    for (int i = 0; i < 4; ++i) hd.pad[i] = 0;
     *p.header = hd;
   }
 }

@@ -18,7 +18,8 @@ struct PlanHeader {
   int32_t n_items;
   int32_t chunk_len;
   int32_t partial_floats;
-  int32_t pad[5];
+  int32_t next_item;   // work counter of the persistent attention kernel (zeroed by the planner)
+  int32_t pad[4];
 };
 
 constexpr int kItemsPerSM = 4;     // target work items per SM for split-KV
@@ -34,6 +35,7 @@ struct Layout {
   size_t plan_header = 0;     // PlanHeader
   size_t req_item_begin = 0;  // int32 [B]  first item of request r
   size_t req_chunks = 0;      // int32 [B]  chunks per KV head of request r
+  size_t pair_done = 0;       // int32 [B * Hkv] finished chunks per split (request, head)
   size_t items = 0;           // WorkItem [max_items]
   size_t partials = 0;        // float [partial_cap]
   size_t total = 0;
@@ -53,7 +55,7 @@ struct PlanParams {
   DeviceStatus *status;
   int32_t *q_row_start, *draft_start, *req_flag;
   PlanHeader *header;
-  int32_t *req_item_begin, *req_chunks;
+  int32_t *req_item_begin, *req_chunks, *pair_done;
   WorkItem *items;
 };
 

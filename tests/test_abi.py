@@ -76,7 +76,7 @@ BAD_ATTN = [dict(B=-1), dict(Hq=0), dict(Hq=6, Hkv=4), dict(D=96), dict(block_si
             dict(q=None), dict(out=0x40004), dict(qkv_dtype=7), dict(total_q_rows=1), dict(num_blocks=0),
             dict(max_blocks_per_seq=0)]
 BAD_ACC = [dict(B=-2), dict(V=0), dict(total_draft=-1), dict(target_logits=None), dict(draft_probs=None),
-           dict(logits_dtype=3), dict(total_q_rows=1), dict(V=10_000_000), dict(next_token=None)]
+           dict(logits_dtype=3), dict(total_q_rows=1), dict(V=(1 << 24) + 1), dict(next_token=None)]
 
 
 @pytest.mark.parametrize("kw", BAD_ATTN, ids=[str(k) for k in BAD_ATTN])
