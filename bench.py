@@ -257,6 +257,9 @@ def run_ours(args, batch, rank, world, local_rank):
     ms = _time_loop(db.step, args.steps, flush, torch)
     clocks = sampler.stop() if sampler else None
     torch.cuda.synchronize()
+    code, rid = db.device_status()
+    if code != 0:
+        raise RuntimeError(f"device status {code} at request {rid} after the timed steps")
     total_ms = sum(ms)
     verified_all = verified
     if world > 1:

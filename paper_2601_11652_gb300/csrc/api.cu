@@ -113,6 +113,7 @@ Layout make_layout(const wisp_attn_args *a, const wisp_accept_args *c, int sms) 
     L.req_chunks = take(sizeof(int32_t) * (size_t)B);
     L.pair_done = take(sizeof(int32_t) * (size_t)B * a->Hkv);
     L.items = take(sizeof(WorkItem) * (size_t)L.max_items);
+    L.order = take(sizeof(int32_t) * (size_t)L.max_items);
     L.partials = take(sizeof(float) * (size_t)L.partial_cap);
   }
   L.total = off;
@@ -157,6 +158,7 @@ PlanParams plan_params(const wisp_attn_args *a, const wisp_accept_args *c, void 
     pp.req_chunks = at<int32_t>(ws, L.req_chunks);
     pp.pair_done = at<int32_t>(ws, L.pair_done);
     pp.items = at<WorkItem>(ws, L.items);
+    pp.order = at<int32_t>(ws, L.order);
   } else {
     pp.Hq = pp.Hkv = 1;
   }
@@ -184,6 +186,7 @@ wisp_status launch_attention(const wisp_attn_args *a, void *ws, const Layout &L,
   ap.header = at<PlanHeader>(ws, L.plan_header);
   ap.header_mut = at<PlanHeader>(ws, L.plan_header);
   ap.items = at<WorkItem>(ws, L.items);
+  ap.order = at<int32_t>(ws, L.order);
   ap.partials = at<float>(ws, L.partials);
   ap.pair_done = at<int32_t>(ws, L.pair_done);
   const bool bf = a->qkv_dtype == WISP_BF16;

@@ -16,6 +16,7 @@ struct AttnParams {
   const PlanHeader *header;
   PlanHeader *header_mut;  // same object: the work counter
   const WorkItem *items;
+  const int32_t *order;  // dispatch order of the persistent kernel: item index per counter value
   float *partials;
   int32_t *pair_done;  // [B * Hkv] finished chunks of each split (request, head), zeroed by the planner
 };

@@ -13,6 +13,8 @@ namespace wisp {
 namespace {
 
 constexpr int kThreads = 1024;
+constexpr int kOrderBuckets = 1024;  // tile-count buckets of the dispatch order
+constexpr int kOrderTile = 64;       // tokens per KV tile of the attention kernels
 
 __device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
 __device__ __forceinline__ int64_t max64(int64_t a, int64_t b) { return a > b ? a : b; }
@@ -151,9 +153,33 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     item_carry += ti;
     poff_carry += tp;
   }
+  // pass 4: dispatch order, longest items first (counting sort on the tile count), so that the
+  // persistent kernel ends with its shortest items and its CTAs finish close together
+  __shared__ int32_t s_hist[kOrderBuckets];
+  const int64_t n_items = min64(item_carry, p.max_items);
+  for (int b = tid; b < kOrderBuckets; b += kThreads) s_hist[b] = 0;
+  __syncthreads();  // also makes pass 3's items visible to every thread of the block
+  auto bucket = [&](int64_t i) -> int {
+    const WorkItem &w = p.items[i];
+    const int64_t tiles = ((int64_t)w.t1 - w.t0 + kOrderTile - 1) / kOrderTile;
+    return kOrderBuckets - 1 - (int)max64(0, min64(tiles, kOrderBuckets - 1));  // bucket 0: the longest
+  };
+  for (int64_t i = tid; i < n_items; i += kThreads) atomicAdd(&s_hist[bucket(i)], 1);
+  __syncthreads();
+  {
+    static_assert(kOrderBuckets == kThreads, "one bucket per thread in the scan");
+    int64_t tot;
+    const int64_t incl = block_scan(s_hist[tid], s_warp, &tot);
+    const int32_t excl = (int32_t)(incl - s_hist[tid]);
+    __syncthreads();
+    s_hist[tid] = excl;
+    __syncthreads();
+  }
+  for (int64_t i = tid; i < n_items; i += kThreads) p.order[atomicAdd(&s_hist[bucket(i)], 1)] = (int32_t)i;
+
   if (tid == 0) {
     PlanHeader hd;
-    hd.n_items = (int32_t)min64(item_carry, p.max_items);
+    hd.n_items = (int32_t)n_items;
     hd.chunk_len = (int32_t)chunk;
     hd.partial_floats = (int32_t)min64(poff_carry, p.partial_cap);
     hd.next_item = 0;

@@ -37,6 +37,7 @@ struct Layout {
   size_t req_chunks = 0;      // int32 [B]  chunks per KV head of request r
   size_t pair_done = 0;       // int32 [B * Hkv] finished chunks per split (request, head)
   size_t items = 0;           // WorkItem [max_items]
+  size_t order = 0;           // int32 [max_items]  dispatch order of the items (largest first)
   size_t partials = 0;        // float [partial_cap]
   size_t total = 0;
   int64_t max_items = 0;
@@ -57,6 +58,7 @@ struct PlanParams {
   PlanHeader *header;
   int32_t *req_item_begin, *req_chunks, *pair_done;
   WorkItem *items;
+  int32_t *order;
 };
 
 __global__ void plan_kernel(const PlanParams p);
