@@ -163,6 +163,20 @@ wisp_status wisp_verify_accept(const wisp_accept_args *acc, void *workspace, siz
 wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args *acc, void *workspace,
                              size_t workspace_bytes, void *stream);
 
+/* Acceptance pass (same rule, kernels and results as wisp_verify_accept) that needs no workspace
+ * and allocates nothing.  No counterpart in the paper: it exists for callers that cannot allocate
+ * device memory when they verify (memory owned by another allocator, or a latency path on which
+ * cudaMalloc, which may synchronise the device, is not allowed).
+ *   Scratch: a fixed 128 KiB array inside this library's device image, shared by every call in
+ *   the process.  Calls that overlap in time (other streams, other host threads) race on it and
+ *   corrupt each other's results: order them, e.g. on one stream.
+ *   Limit: B <= 8192 requests; a larger batch returns WISP_ERR_UNSUPPORTED and enqueues nothing.
+ *   Set-up: the first call on a device looks up the array's address and sets kernel attributes
+ *   (host-side runtime calls, no allocation); make that first call before any stream capture.
+ *   Device-data errors are recorded in the scratch's status word, which this entry point does not
+ *   expose; a caller that must read them uses wisp_verify_accept with its own workspace. */
+wisp_status wisp_verify_accept_noalloc(const wisp_accept_args *acc, void *stream);
+
 /* Read the device status word of `workspace` (synchronous copy; synchronise the stream that
  * ran the step first).  *code receives a wisp_device_code, *request_id the request_ids entry
  * (or the batch index when request_ids was NULL) of the first failing request, or -1. */

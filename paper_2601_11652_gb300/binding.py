@@ -73,6 +73,8 @@ def load(path: str | None = None):
     lib.wisp_verify_accept.restype = ctypes.c_int
     lib.wisp_verify_step.argtypes = [AP, CP, _P, ctypes.c_size_t, _P]
     lib.wisp_verify_step.restype = ctypes.c_int
+    lib.wisp_verify_accept_noalloc.argtypes = [CP, _P]
+    lib.wisp_verify_accept_noalloc.restype = ctypes.c_int
     lib.wisp_verify_get_device_status.argtypes = [_P, ctypes.POINTER(_I32), ctypes.POINTER(ctypes.c_int64)]
     lib.wisp_verify_get_device_status.restype = ctypes.c_int
     lib.wisp_verify_status_string.argtypes = [ctypes.c_int]
@@ -174,6 +176,10 @@ def wisp_verify_attention(attn: wisp_attn_args, workspace: torch.Tensor, stream=
 def wisp_verify_accept(acc: wisp_accept_args, workspace: torch.Tensor, stream=None) -> None:
     _check("wisp_verify_accept", load().wisp_verify_accept(
         ctypes.byref(acc), _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def wisp_verify_accept_noalloc(acc: wisp_accept_args, stream=None) -> None:
+    _check("wisp_verify_accept_noalloc", load().wisp_verify_accept_noalloc(ctypes.byref(acc), _stream(stream)))
 
 
 def wisp_verify_step(attn: wisp_attn_args, acc: wisp_accept_args, workspace: torch.Tensor, stream=None) -> None:

@@ -250,6 +250,30 @@ wisp_status launch_plan(const wisp_attn_args *a, const wisp_accept_args *c, void
 
 }  // namespace
 
+// Workspace of wisp_verify_accept_noalloc: status word, per-request offsets and flags, planner
+// header.  128 KiB holds them for batches of up to kNoAllocMaxBatch requests.
+constexpr size_t kNoAllocScratchBytes = 128 << 10;
+constexpr int kNoAllocMaxBatch = 8192;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+namespace {
+
+void *g_noalloc_ptr[kMaxDevices];  // device address of g_noalloc_scratch, per device
+
+// Address of the scratch array on the current device `dev`, looked up once (under g_mu).
+wisp_status noalloc_scratch(int dev, void **out) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void *ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return WISP_ERR_CUDA;
+    g_noalloc_ptr[dev] = ptr;
+  }
+  *out = g_noalloc_ptr[dev];
+  return WISP_OK;
+}
+
+}  // namespace
+
 extern "C" {
 
 size_t wisp_verify_workspace_size(const wisp_attn_args *attn, const wisp_accept_args *acc) {
@@ -312,6 +336,31 @@ wisp_status wisp_verify_get_device_status(const void *ws, int32_t *code, int64_t
   *code = h.code;
   *request_id = h.code ? h.request_id : -1;
   return WISP_OK;
+}
+
+// ---- acceptance pass without a caller workspace (no counterpart in the paper) -----------------
+// Some callers cannot allocate device memory when they verify: a serving loop whose memory is
+// owned by another allocator (a caching pool it must not bypass), or a latency path where
+// cudaMalloc is off limits because it can synchronise the device.  This entry point runs the same
+// planner and acceptance kernels as wisp_verify_accept, with their workspace carved from a fixed
+// array in this library's device image instead of caller memory.  Nothing here allocates: the
+// array exists once the module is loaded, and the first call on a device only looks up its
+// address (cudaGetSymbolAddress) and sets kernel attributes.
+wisp_status wisp_verify_accept_noalloc(const wisp_accept_args *acc, void *stream) {
+  wisp_status st = check_accept(acc);
+  if (st != WISP_OK) return st;
+  if (acc->B > kNoAllocMaxBatch) return WISP_ERR_UNSUPPORTED;  // beyond the fixed scratch
+  int dev = 0, sms = 0;
+  if ((st = device_setup(&dev, &sms)) != WISP_OK) return st;
+  const Layout L = make_layout(nullptr, acc, sms);
+  if (L.total > kNoAllocScratchBytes) return WISP_ERR_UNSUPPORTED;
+  void *ws = nullptr;
+  if ((st = noalloc_scratch(dev, &ws)) != WISP_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the planner clears the status word (the only field that must start at zero) on `s` first
+  if ((st = launch_plan(nullptr, acc, ws, L, s)) != WISP_OK) return st;
+  if (acc->B == 0) return WISP_OK;
+  return launch_accept(acc, ws, L, sms, s);
 }
 
 const char *wisp_verify_status_string(wisp_status s) {
