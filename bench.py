@@ -58,6 +58,12 @@ def accept_bytes(b, L) -> int:
     return rows + qrow + gathers + b.B * 16
 
 
+def _launches_per_step(b) -> int:
+    """Kernels of this library one wisp_verify_step launches: planner, attention (tensor-core
+    kernel for bf16; SIMT kernel + combine for fp32), acceptance."""
+    return 3 if b.dtype == "bf16" else 4
+
+
 def _peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -301,7 +307,7 @@ def run_ours(args, batch, rank, world, local_rank):
             "emitted_tokens_per_s": (verified_all + batch.B * world) / (ms_per_step / 1e3),
             "mean_acceptance": float(verified / max(1, batch.total_draft)),
             "cpu_baseline": cpu_baseline(batch),
-            "e2e": e2e, "gpu_launches": 4 * args.steps, "clocks": clocks}
+            "e2e": e2e, "gpu_launches": _launches_per_step(batch) * args.steps, "clocks": clocks}
     print(json.dumps(line), flush=True)
 
 
