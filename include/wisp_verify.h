@@ -159,7 +159,10 @@ wisp_status wisp_verify_accept(const wisp_accept_args *acc, void *workspace, siz
                                void *stream);
 
 /* Enqueue one whole verification step (Sec. 4.5): attention and acceptance.  The two parts
- * read disjoint inputs; draft_lens must describe the same batch in both structs. */
+ * read disjoint inputs; draft_lens must describe the same batch in both structs.  Part of the
+ * acceptance pass (its row statistics) runs on a stream owned by the library, forked from and
+ * joined back into `stream` with events, so work queued on `stream` afterwards sees the whole
+ * step finished. */
 wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args *acc, void *workspace,
                              size_t workspace_bytes, void *stream);
 
@@ -167,10 +170,11 @@ wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args 
  * and allocates nothing.  No counterpart in the paper: it exists for callers that cannot allocate
  * device memory when they verify (memory owned by another allocator, or a latency path on which
  * cudaMalloc, which may synchronise the device, is not allowed).
- *   Scratch: a fixed 128 KiB array inside this library's device image, shared by every call in
+ *   Scratch: a fixed 4 MiB array inside this library's device image, shared by every call in
  *   the process.  Calls that overlap in time (other streams, other host threads) race on it and
  *   corrupt each other's results: order them, e.g. on one stream.
- *   Limit: B <= 8192 requests; a larger batch returns WISP_ERR_UNSUPPORTED and enqueues nothing.
+ *   Limit: B <= 8192 requests and total_q_rows <= 131072; a larger batch returns
+ *   WISP_ERR_UNSUPPORTED and enqueues nothing.
  *   Set-up: the first call on a device looks up the array's address and sets kernel attributes
  *   (host-side runtime calls, no allocation); make that first call before any stream capture.
  *   Device-data errors are recorded in the scratch's status word, which this entry point does not

@@ -1,23 +1,27 @@
 // accept.cu -- the in-order speculative acceptance pass over the vocabulary (Eq. 1-3).
 //
-// One thread-block cluster of C CTAs (C = 1..8, chosen from the batch size) serves one
-// request; CTA c owns a contiguous slice of every logit row, streamed as 16-byte vectors.
+// Two launches.
 //
-// Walk (Eq. 1-2): for logit rows i = 0, 1, ... of the request (row i scores draft token
-// i+1; row k is the bonus row):
-//   * one streaming pass gives each thread a running max and a double-float running sum
-//     of exp(z - max) (fp32 terms, pairwise within a vector); threads, then CTAs (through
-//     distributed shared memory, in rank order so every CTA holds bit-identical values)
-//     combine them.  Alongside, a certified bound on the relative error of the normaliser
-//     Z is accumulated (fp32 exp error, rounding of z - m, every rescale, pairwise sums);
-//   * the decision u_i <= min(1, p(y)/q(y)) is taken in fp32 when u_i lies outside the
-//     certified interval of the ratio; otherwise Z and p(y) are recomputed in double-float
-//     arithmetic (Tang's table-driven exp) and the decision is taken on those;
-//   * the walk stops at the first rejection, so later rows are never read.
-// Draw (Eq. 3): from max(0, p_L - q_{L+1}) after a rejection, else from p_L, by inverse
-// CDF in ascending token order: one double-float sweep of the row gives per-(round, warp)
-// tile sums in shared memory and per-CTA totals; the CTA holding the crossing of
-// u * total scans its tiles, then one warp scans the tile, then one lane its elements.
+// row_stats_kernel: warp (row, slice) streams one vocabulary slice of one logit row once, as
+// 16-byte vectors; every lane keeps a running max, a double-float running sum of exp(z - max)
+// (fp32 terms, pairwise within a vector) and the terms of a certified bound on the relative
+// error of the normaliser Z (exp error, rounding of the argument, every rescale, pairwise sums);
+// the warp merges them into the slice's statistics.  Every row of the batch is processed, in
+// parallel, so the pass runs at HBM bandwidth; rows past a request's first rejection are read
+// although the rule never uses them.
+//
+// accept_kernel: one thread-block cluster of C CTAs (C = 1..8, chosen from the batch size) per
+// request.  Walk (Eq. 1-2): warp w merges the slice statistics of row i0 + w (rows in batches
+// of 8; row i scores draft token i+1, row k is the bonus row) and thread 0 takes the decisions
+// u_i <= min(1, p(y)/q(y)) in order, in fp32 when u_i lies outside the certified interval of the
+// ratio; otherwise the cluster recomputes that row's Z and p(y) in double-float arithmetic
+// (Tang's table-driven exp) and decides on those.  The walk stops at the first rejection.
+// Draw (Eq. 3): from max(0, p_L - q_{L+1}) after a rejection, else from p_L, by inverse CDF in
+// ascending token order: CTA c owns a contiguous slice of the row; one double-float sweep gives
+// per-(round, warp) tile sums in shared memory and per-CTA totals (through distributed shared
+// memory, summed in rank order so every CTA holds bit-identical values); the CTA holding the
+// crossing of u * total scans its tiles, then one warp scans the tile, then one lane its
+// elements.
 #include <cooperative_groups.h>
 #include <cstring>
 
@@ -114,9 +118,6 @@ __device__ __forceinline__ ff draw_weight(float z, float m, bool residual, float
   return e;
 }
 
-__device__ __forceinline__ void prefetch_l2(const void *p, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-}
 
 // Per-thread streaming statistics of one row slice (see the file comment).
 struct RowStats {
@@ -142,7 +143,7 @@ __device__ __forceinline__ void stats_rebase(RowStats &st, float mnew) {
     return;
   }
   if (!(mnew > st.m)) return;
-  const float f = expf(st.m - mnew);
+  const float f = ex2_approx((st.m - mnew) * kLog2e);
   const float d = mnew - st.m;
   st.s = ff_mul_f(st.s, f);
   st.A = fmaf(st.A, f, d * st.s.hi);
@@ -150,45 +151,43 @@ __device__ __forceinline__ void stats_rebase(RowStats &st, float mnew) {
   st.nres += 1;
 }
 
-template <typename LT>
-__device__ __forceinline__ void stats_add_vec(RowStats &st, const uint4 &w) {
+// Add one chunk of NV vectors (a thread's next elements of its slice): the chunk max first (one
+// rescale at most per chunk), then exp(z - m) = 2^((z - m) * log2 e) per element, a pairwise fp32
+// sum of the chunk added to the double-float running sum, and the bound term A.
+template <typename LT, int NV>
+__device__ __forceinline__ void stats_add_chunk(RowStats &st, const uint4 (&w)[NV]) {
   constexpr int E = LTraits<LT>::E;
-  float z[E];
-  float vm = -INFINITY;
+  constexpr int N = NV * E;
+  float z[N];
 #pragma unroll
-  for (int i = 0; i < E; ++i) {
-    z[i] = vec_elem<LT>(w, i);
-    vm = fmaxf(vm, z[i]);
+  for (int u = 0; u < NV; ++u) {
+#pragma unroll
+    for (int i = 0; i < E; ++i) z[u * E + i] = vec_elem<LT>(w[u], i);
   }
-  if (vm == -INFINITY) return;  // nothing but padding (or -inf logits)
-  if (st.m == -INFINITY) st.mfirst = vm;
-  stats_rebase(st, vm);
-  float e[E];
+  float mx[8];
 #pragma unroll
-  for (int i = 0; i < E; ++i) {
+  for (int i = 0; i < 8; ++i) mx[i] = z[i];
+#pragma unroll
+  for (int i = 8; i < N; ++i) mx[i & 7] = fmaxf(mx[i & 7], z[i]);
+  const float cm = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+  if (cm == -INFINITY) return;  // nothing but padding (or -inf logits)
+  if (st.m == -INFINITY) st.mfirst = cm;
+  stats_rebase(st, cm);
+  float e[N];
+  float a[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+  for (int i = 0; i < N; ++i) {
     const float x = z[i] - st.m;
-    e[i] = expf(x);
-    st.A = fmaf(e[i], fminf(-x, 104.0f), st.A);
+    e[i] = ex2_approx(x * kLog2e);
+    a[i & 3] = fmaf(e[i], fminf(-x, 104.0f), a[i & 3]);
   }
 #pragma unroll
-  for (int w2 = 1; w2 < E; w2 <<= 1) {
+  for (int w2 = 1; w2 < N; w2 <<= 1) {
 #pragma unroll
-    for (int i = 0; i < E; i += 2 * w2) e[i] += e[i + w2];
+    for (int i = 0; i < N; i += 2 * w2) e[i] += e[i + w2];
   }
   st.s = ff_add_f(st.s, e[0]);
-}
-
-// Combine `o` into `st` (both may be empty).
-__device__ __forceinline__ void stats_merge(RowStats &st, const RowStats &o) {
-  if (o.m == -INFINITY) return;
-  RowStats b = o;
-  const float mm = fmaxf(st.m, b.m);
-  stats_rebase(st, mm);
-  stats_rebase(b, mm);
-  st.s = ff_add(st.s, b.s);
-  st.A += b.A;
-  st.nres = max(st.nres, b.nres);
-  st.mfirst = fminf(st.mfirst, b.mfirst);
+  st.A += (a[0] + a[1]) + (a[2] + a[3]);
 }
 
 struct Decide {
@@ -196,7 +195,110 @@ struct Decide {
   float zy, qy, u;
 };
 
+// Warp-wide merge of the S <= 32 slice statistics of one row (lane q reads slice q): the same
+// max / rebase / tree-sum, so every lane (and every CTA that does it) holds identical values.
+// The slice-to-row rebase is not counted in nres; the decision bound allows for it.
+__device__ __forceinline__ RowStats merge_parts(const RowPart *parts, int S) {
+  const int lane = threadIdx.x & 31;
+  RowStats q;
+  stats_init(q);
+  if (lane < S) {
+    const RowPart t = parts[lane];
+    q.m = t.m;
+    q.s = {t.s_hi, t.s_lo};
+    q.A = t.A;
+    q.mfirst = t.mfirst;
+    q.nres = t.nres;
+  }
+  float gm = q.m, gf = q.mfirst;
+  int gn = q.nres;
+  for (int o = 16; o > 0; o >>= 1) {
+    gm = fmaxf(gm, __shfl_xor_sync(0xffffffffu, gm, o));
+    gf = fminf(gf, __shfl_xor_sync(0xffffffffu, gf, o));
+    gn = max(gn, __shfl_xor_sync(0xffffffffu, gn, o));
+  }
+  if (q.m > -INFINITY) stats_rebase(q, gm);
+  ff gs = q.m > -INFINITY ? q.s : ff{0.0f, 0.0f};
+  float ga = q.m > -INFINITY ? q.A : 0.0f;
+  for (int o = 16; o > 0; o >>= 1) {
+    gs = ff_add(gs, ff_shfl_xor(gs, o));
+    ga += __shfl_xor_sync(0xffffffffu, ga, o);
+  }
+  RowStats r;
+  r.m = gm;
+  r.s = gs;
+  r.A = ga;
+  r.nres = gn;
+  r.mfirst = gf;
+  return r;
+}
+
 }  // namespace
+
+// Statistics of one vocabulary slice of one logit row (Eq. 1 needs p = softmax of the row):
+// warp (row, slice) streams its slice once, every lane keeping a running max, a double-float sum
+// of exp(z - m) and the error terms over chunks of 4 vectors (the next chunk's loads are issued
+// before the current one is reduced); the lanes are merged with shuffles (max, rebase, tree sum)
+// and lane 0 writes the slice's statistics.  No shared memory, no block barrier.
+template <typename LT>
+__global__ void __launch_bounds__(NT) row_stats_kernel(const __grid_constant__ AcceptParams p) {
+  constexpr int E = LTraits<LT>::E;
+  const int lane = threadIdx.x & 31;
+  const int64_t unit = (int64_t)blockIdx.x * NW + (threadIdx.x >> 5);
+  if (unit >= p.total_rows * p.slices) return;
+  const int64_t row = unit / p.slices;
+  const int sl = (int)(unit % p.slices);
+  const int V = p.V;
+  const LT *rowp = static_cast<const LT *>(p.logits) + row * (int64_t)V;
+  const bool vec_z = p.vec_z != 0;
+  const int64_t nvec = (V + E - 1) / E;
+  const int64_t vlo = min(nvec, (int64_t)sl * p.vps);
+  const int64_t vhi = min(nvec, vlo + p.vps);
+  const uint32_t ni = LTraits<LT>::NEG_INF2;
+  auto load4 = [&](int64_t base, uint4 (&w)[4]) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t vi = base + u * 32;
+      w[u] = vi < vhi ? load_vec<LT>(rowp, vi, V, vec_z) : make_uint4(ni, ni, ni, ni);
+    }
+  };
+  RowStats st;
+  stats_init(st);
+  uint4 cur[4];
+  load4(vlo + lane, cur);
+  for (int64_t base = vlo + lane; base < vhi; base += 4 * 32) {
+    uint4 nxt[4];
+    load4(base + 4 * 32, nxt);
+    stats_add_chunk<LT, 4>(st, cur);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) cur[u] = nxt[u];
+  }
+  // lanes -> slice: max, rebase, tree sum (the lane-to-slice rebase counts as one more rescale)
+  float wm = st.m, wf = st.mfirst;
+  int wn = st.nres;
+  for (int o = 16; o > 0; o >>= 1) {
+    wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
+    wf = fminf(wf, __shfl_xor_sync(0xffffffffu, wf, o));
+    wn = max(wn, __shfl_xor_sync(0xffffffffu, wn, o));
+  }
+  if (wm > -INFINITY) stats_rebase(st, wm);
+  ff ws = st.m > -INFINITY ? st.s : ff{0.0f, 0.0f};
+  float wa = st.m > -INFINITY ? st.A : 0.0f;
+  for (int o = 16; o > 0; o >>= 1) {
+    ws = ff_add(ws, ff_shfl_xor(ws, o));
+    wa += __shfl_xor_sync(0xffffffffu, wa, o);
+  }
+  if (lane == 0) {
+    RowPart out;
+    out.m = wm;
+    out.s_hi = ws.hi;
+    out.s_lo = ws.lo;
+    out.A = wa;
+    out.mfirst = wf;
+    out.nres = wn + 1;
+    p.parts[unit] = out;
+  }
+}
 
 template <typename LT>
 __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ AcceptParams p) {
@@ -204,9 +306,10 @@ __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ Acce
   extern __shared__ ff s_tile[];  // [rounds * NW] per-(round, warp) draw sums
   __shared__ float s_th[256], s_tl[256];
   __shared__ RowStats s_wst[NW];
-  __shared__ RowStats s_pub[2];   // this CTA's published statistics (ring of 2)
-  __shared__ ff s_tot[8];
-  __shared__ RowStats s_row;      // combined statistics of the current row
+  __shared__ RowStats s_pub[2];   // this CTA's published totals (ring of 2)
+  __shared__ ff s_tot[kMaxAcceptCluster];
+  __shared__ RowStats s_rows[NW]; // merged statistics of the rows being walked
+  __shared__ int s_walk[2];       // walk state, row within the batch
   __shared__ float s_zy[kPreload], s_qy[kPreload], s_u[kPreload];
   __shared__ Decide s_dec;
   __shared__ int s_bad;
@@ -251,89 +354,7 @@ __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ Acce
   }
   __syncthreads();
 
-  // ---- reductions -----------------------------------------------------------
-  // CTA-wide merge of per-thread statistics (max first, then every thread rebases to it and
-  // the sums are tree-reduced), then the cluster-wide merge: lane q of warp 0 reads CTA q's
-  // published statistics and the same max / rebase / tree-sum runs across those lanes, so
-  // every CTA ends with bit-identical values.
-  auto cluster_stats = [&](RowStats st) -> RowStats {
-    float wm = st.m, wf = st.mfirst;
-    int wn = st.nres;
-    for (int o = 16; o > 0; o >>= 1) {
-      wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
-      wf = fminf(wf, __shfl_xor_sync(0xffffffffu, wf, o));
-      wn = max(wn, __shfl_xor_sync(0xffffffffu, wn, o));
-    }
-    if (lane == 0) {
-      s_wst[warp].m = wm;
-      s_wst[warp].mfirst = wf;
-      s_wst[warp].nres = wn;
-    }
-    __syncthreads();
-    float cm = -INFINITY, cf = INFINITY;
-    int cn = 0;
-    for (int w = 0; w < NW; ++w) {
-      cm = fmaxf(cm, s_wst[w].m);
-      cf = fminf(cf, s_wst[w].mfirst);
-      cn = max(cn, s_wst[w].nres);
-    }
-    if (cm > -INFINITY) stats_rebase(st, cm);
-    ff ws = st.s;
-    float wa = st.A;
-    for (int o = 16; o > 0; o >>= 1) {
-      ws = ff_add(ws, ff_shfl_xor(ws, o));
-      wa += __shfl_xor_sync(0xffffffffu, wa, o);
-    }
-    __syncthreads();  // everyone has read s_wst[*].m
-    if (lane == 0) {
-      s_wst[warp].s = ws;
-      s_wst[warp].A = wa;
-    }
-    __syncthreads();
-    if (tid == 0) {
-      RowStats c;
-      c.m = cm;
-      c.mfirst = cf;
-      c.nres = cn + 1;  // the thread-to-CTA rebase
-      c.s = {0.0f, 0.0f};
-      c.A = 0.0f;
-      for (int w = 0; w < NW; ++w) {
-        c.s = ff_add(c.s, s_wst[w].s);
-        c.A += s_wst[w].A;
-      }
-      s_pub[xslot] = c;
-    }
-    cluster.sync();
-    if (warp == 0) {
-      RowStats q;
-      stats_init(q);
-      if (lane < C) q = *cluster.map_shared_rank(&s_pub[xslot], lane);
-      float gm = q.m, gf = q.mfirst;
-      int gn = q.nres;
-      for (int o = 16; o > 0; o >>= 1) {
-        gm = fmaxf(gm, __shfl_xor_sync(0xffffffffu, gm, o));
-        gf = fminf(gf, __shfl_xor_sync(0xffffffffu, gf, o));
-        gn = max(gn, __shfl_xor_sync(0xffffffffu, gn, o));
-      }
-      if (q.m > -INFINITY) stats_rebase(q, gm);
-      ff gs = q.m > -INFINITY ? q.s : ff{0.0f, 0.0f};
-      float ga = q.m > -INFINITY ? q.A : 0.0f;
-      for (int o = 16; o > 0; o >>= 1) {
-        gs = ff_add(gs, ff_shfl_xor(gs, o));
-        ga += __shfl_xor_sync(0xffffffffu, ga, o);
-      }
-      if (lane == 0) {
-        s_row.m = gm;
-        s_row.s = gs;
-        s_row.A = ga;
-        s_row.nres = gn;  // + the CTA-to-cluster rebase, counted in the bound
-        s_row.mfirst = gf;
-      }
-    }
-    __syncthreads();
-    xslot ^= 1;
-    return s_row;
-  };
+  // ---- reductions across the cluster -----------------------------------------------
   // ff total over the CTA (per-thread values), every CTA's total gathered into s_tot,
   // and their sum in rank order
   auto cluster_total = [&](ff a) -> ff {
@@ -368,98 +389,111 @@ __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ Acce
   };
 
   // ---- the in-order walk (Eq. 1-2) -------------------------------------------
+  // The rows' statistics come from row_stats_kernel: warp w merges the slices of row i0 + w,
+  // then thread 0 takes the decisions of the batch in order; a decision inside the certified
+  // interval of the fp32 ratio stops it, the whole cluster recomputes that row's normaliser in
+  // double-float arithmetic, and the walk resumes after it.
   int L = k;
   int err = s_bad ? WISP_DEV_BAD_TOKEN : 0;
   float m = 0.0f;
   ff Zff = {0.0f, 0.0f};
   bool have_Zff = false;
-  for (int i = 0; i <= k && !err; ++i) {
-    const LT *row = logits + (Q0 + i) * (int64_t)V;
-    if (p.prefetch && i < k && tid == 0 && vhi > vlo) {
-      const LT *nrow = row + V;
-      const uint64_t a0 = reinterpret_cast<uint64_t>(nrow + vlo * E) & ~uint64_t(15);
-      const uint64_t a1 = reinterpret_cast<uint64_t>(nrow + min((int64_t)V, vhi * E)) & ~uint64_t(15);
-      for (uint64_t a = a0; a < a1; a += 32768) {
-        const uint64_t n = a1 - a < 32768 ? a1 - a : 32768;
-        prefetch_l2(reinterpret_cast<const void *>(a), (uint32_t)n);
-      }
-    }
-    RowStats st;
-    stats_init(st);
-    for (int64_t base = vlo + tid; base < vhi; base += 4 * NT) {
-      uint4 w[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int64_t vi = base + u * NT;
-        const uint32_t ni = LTraits<LT>::NEG_INF2;
-        w[u] = vi < vhi ? load_vec<LT>(row, vi, V, vec_z) : make_uint4(ni, ni, ni, ni);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) stats_add_vec<LT>(st, w[u]);
-    }
-    const RowStats rs = cluster_stats(st);
-    m = rs.m;
-    const ff Z = rs.s;
-    have_Zff = false;
-    if (!(m > -INFINITY) || !(m < INFINITY) || !(Z.hi > 0.0f) || !(Z.hi < INFINITY) || !(rs.A >= 0.0f)) {
-      err = WISP_DEV_BAD_PROB;
-      break;
-    }
-    if (i == k) break;  // bonus row reached: every draft token accepted
-
-    // Eq. 1, taken identically by thread 0 of every CTA
-    if (tid == 0) {
-      Decide d;
-      if (i < kPreload) {
-        d.zy = s_zy[i];
-        d.qy = s_qy[i];
-        d.u = s_u[i];
-      } else {
-        const int32_t y = __ldg(p.draft_tokens + D0 + i);
-        d.zy = load_scalar(row, y);
-        d.qy = __ldg(p.draft_probs + (D0 + i) * (int64_t)V + y);
-        d.u = __ldg(p.accept_u + D0 + i);
-      }
-      if (!(d.qy >= 0.0f)) {
-        d.flag = 4;
-      } else if (d.qy == 0.0f) {
-        d.flag = 0;  // a = 1
-      } else {
-        // certified relative error of Z (see RowStats) and of the ratio p(y)/q(y)
-        const float x = d.zy - m;
-        const float dz = 1.05f * ((float)(rs.nres + 2) * 0x1p-22f + 0x1p-24f * (m - rs.mfirst) +
-                                  0x1p-24f * (rs.A / Z.hi) + 4.0f * 0x1p-24f) +
-                         1e-12f;
-        const float dr = dz + 1.05f * (0x1p-22f + 0x1p-24f * fabsf(x) + 4.0f * 0x1p-24f);
-        const float ratio = expf(x) / (Z.hi * d.qy);
-        const float lo = fminf(1.0f, ratio * (1.0f - dr)), hi = fminf(1.0f, ratio * (1.0f + dr));
-        d.flag = d.u <= lo ? 0 : (d.u > hi ? 1 : 2);
-      }
-      s_dec = d;
+  bool done = err != 0;
+  const int nsl = p.slices;
+  for (int i0 = 0; i0 <= k && !done; i0 += NW) {
+    if (i0 + warp <= k) {
+      const RowStats rs = merge_parts(p.parts + (Q0 + i0 + warp) * (int64_t)nsl, nsl);
+      if (lane == 0) s_rows[warp] = rs;
     }
     __syncthreads();
-    Decide d = s_dec;
-    if (d.flag == 4) {
-      err = WISP_DEV_BAD_PROB;
-      break;
-    }
-    if (d.flag == 2) {
-      // inside the certified interval: decide with the double-float normaliser
-      Zff = row_Zff(row, m);
-      have_Zff = true;
+    int j = 0;
+    while (!done) {
       if (tid == 0) {
-        const ff x = ff_two_sum(d.zy, -m);
-        const ff e = ff_exp_nonpos(x.hi, x.lo, s_th, s_tl);
-        const double ratio = ff_to_double(e) / (ff_to_double(Zff) * (double)d.qy);
-        s_dec.flag = (double)d.u <= fmin(1.0, ratio) ? 0 : 1;
+        // state: 0 batch exhausted, 1 bonus row reached, 2 rejected, 3 bad row, 4 uncertain
+        int state = 0, jj = j;
+        Decide d;
+        d.flag = 0;
+        for (; jj < NW && i0 + jj <= k; ++jj) {
+          const int i = i0 + jj;
+          const RowStats rs = s_rows[jj];
+          const float mi = rs.m;
+          const ff Z = rs.s;
+          if (!(mi > -INFINITY) || !(mi < INFINITY) || !(Z.hi > 0.0f) || !(Z.hi < INFINITY) || !(rs.A >= 0.0f)) {
+            state = 3;
+            break;
+          }
+          if (i == k) {
+            state = 1;  // every draft token accepted
+            break;
+          }
+          if (i < kPreload) {
+            d.zy = s_zy[i];
+            d.qy = s_qy[i];
+            d.u = s_u[i];
+          } else {
+            const int32_t y = __ldg(p.draft_tokens + D0 + i);
+            d.zy = load_scalar(logits + (Q0 + i) * (int64_t)V, y);
+            d.qy = __ldg(p.draft_probs + (D0 + i) * (int64_t)V + y);
+            d.u = __ldg(p.accept_u + D0 + i);
+          }
+          if (!(d.qy >= 0.0f)) {
+            state = 3;
+            break;
+          }
+          if (d.qy == 0.0f) continue;  // a = 1: accepted
+          // certified relative error of Z (see RowStats) and of the ratio p(y)/q(y)
+          // terms: one exp error per element and per rescale on its way (thread, CTA, row), three
+          // roundings in the argument (z - m, log2 e, the product) of every element and every
+          // rescale, the 32-term pairwise sums; the decision's own exp and ratio on top
+          const float x = d.zy - mi;
+          const float dz = 1.05f * ((float)(rs.nres + 2) * kEx2RelErr + 3.0f * 0x1p-24f * (mi - rs.mfirst) +
+                                    3.0f * 0x1p-24f * (rs.A / Z.hi) + 6.0f * 0x1p-24f) +
+                           1e-12f;
+          const float dr = dz + 1.05f * (kEx2RelErr + 3.0f * 0x1p-24f * fabsf(x) + 4.0f * 0x1p-24f);
+          const float ratio = ex2_approx(x * kLog2e) / (Z.hi * d.qy);
+          const float lo = fminf(1.0f, ratio * (1.0f - dr)), hi = fminf(1.0f, ratio * (1.0f + dr));
+          if (d.u <= lo) continue;
+          state = d.u > hi ? 2 : 4;
+          break;
+        }
+        s_walk[0] = state;
+        s_walk[1] = jj;
+        s_dec = d;
       }
       __syncthreads();
-      d.flag = s_dec.flag;
-    }
-    __syncthreads();
-    if (d.flag == 1) {
-      L = i;
-      break;
+      const int state = s_walk[0], jj = s_walk[1];
+      if (state == 0) break;  // next batch
+      if (state == 3) {
+        err = WISP_DEV_BAD_PROB;
+        done = true;
+      } else if (state == 1 || state == 2) {
+        L = i0 + jj;
+        m = s_rows[jj].m;
+        done = true;
+      } else {
+        // inside the certified interval: decide with the double-float normaliser
+        const int i = i0 + jj;
+        const float mi = s_rows[jj].m;
+        const ff zf = row_Zff(logits + (Q0 + i) * (int64_t)V, mi);
+        if (tid == 0) {
+          const Decide d = s_dec;
+          const ff x = ff_two_sum(d.zy, -mi);
+          const ff e = ff_exp_nonpos(x.hi, x.lo, s_th, s_tl);
+          const double ratio = ff_to_double(e) / (ff_to_double(zf) * (double)d.qy);
+          s_walk[0] = (double)d.u <= fmin(1.0, ratio) ? 0 : 1;
+        }
+        __syncthreads();
+        if (s_walk[0] == 1) {
+          L = i;
+          m = mi;
+          Zff = zf;
+          have_Zff = true;
+          done = true;
+        } else {
+          j = jj + 1;  // accepted: resume the walk after this row
+        }
+      }
+      __syncthreads();  // s_walk / s_dec are rewritten by the next round
     }
   }
 
@@ -642,11 +676,24 @@ namespace {
 
 template <typename LT>
 cudaError_t set_attr() {
-  return cudaFuncSetAttribute(accept_kernel<LT>, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
+  // the maximum shared-memory carveout, like the attention kernel, so that these CTAs can share an
+  // SM with an attention CTA when wisp_verify_step runs both at once
+  cudaError_t e = cudaFuncSetAttribute(accept_kernel<LT>, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(accept_kernel<LT>, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(row_stats_kernel<LT>, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
+  return e;
 }
 
 template <typename LT>
-cudaError_t launch_t(const AcceptParams &ap, cudaStream_t s) {
+cudaError_t stats_t(const AcceptParams &ap, cudaStream_t s) {
+  row_stats_kernel<LT><<<(unsigned)((ap.total_rows * ap.slices + NW - 1) / NW), NT, 0, s>>>(ap);
+  return cudaGetLastError();
+}
+
+template <typename LT>
+cudaError_t walk_t(const AcceptParams &ap, cudaStream_t s) {
   const int rounds = (ap.vpc + NT - 1) / NT;
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof cfg);
@@ -672,8 +719,12 @@ cudaError_t accept_setup() {
   return e;
 }
 
-cudaError_t accept_launch(const AcceptParams &p, bool bf16, cudaStream_t s) {
-  return bf16 ? launch_t<uint16_t>(p, s) : launch_t<float>(p, s);
+cudaError_t accept_stats_launch(const AcceptParams &p, bool bf16, cudaStream_t s) {
+  return bf16 ? stats_t<uint16_t>(p, s) : stats_t<float>(p, s);
+}
+
+cudaError_t accept_walk_launch(const AcceptParams &p, bool bf16, cudaStream_t s) {
+  return bf16 ? walk_t<uint16_t>(p, s) : walk_t<float>(p, s);
 }
 
 }  // namespace wisp

@@ -9,12 +9,23 @@ constexpr int kAcceptThreads = 256;  // 8 warps per CTA
 constexpr int kMaxAcceptCluster = 8;
 constexpr int kPreload = 256;        // decision inputs gathered up front for the first rows
 
+// Statistics of one vocabulary slice of one logit row (written by row_stats_kernel): running max,
+// double-float sum of exp(z - m), the error terms of the certified bound, rescale count.
+struct RowPart {
+  float m, s_hi, s_lo, A, mfirst;
+  int nres;
+};
+constexpr int kMaxSlices = 32;  // slices per row (one warp lane each when they are merged)
+
 struct AcceptParams {
   int B, V;
   int cluster;        // CTAs per request (1..8), = cluster size of the launch
   int vpc;            // 16-byte vectors of a row per CTA (multiple of 32)
   int vec_z, vec_q;   // 1 if logit rows / draft-prob rows are 16-byte aligned for vector loads
-  int prefetch;       // 1: prefetch the next logit row into L2 while deciding the current one
+  int slices;         // vocabulary slices per row of row_stats_kernel (1..kMaxSlices)
+  int vps;            // 16-byte vectors per slice (multiple of 32)
+  int64_t total_rows; // logit rows (grid of row_stats_kernel = total_rows * slices)
+  RowPart *parts;     // [total_rows, slices]
   const int64_t *request_ids;
   const int32_t *draft_lens;
   const void *logits;
@@ -28,7 +39,9 @@ struct AcceptParams {
 };
 
 cudaError_t accept_setup();  // once per device: shared-memory attributes
-// rounds = ceil(vpc / kAcceptThreads): sizes the per-(round, warp) draw partials
-cudaError_t accept_launch(const AcceptParams &p, bool bf16, cudaStream_t s);
+// statistics of every logit row (needs only the logits)
+cudaError_t accept_stats_launch(const AcceptParams &p, bool bf16, cudaStream_t s);
+// per-request walk and draw (needs the statistics and the planner's offsets)
+cudaError_t accept_walk_launch(const AcceptParams &p, bool bf16, cudaStream_t s);
 
 }  // namespace wisp

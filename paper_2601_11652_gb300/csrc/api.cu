@@ -16,6 +16,11 @@ constexpr int kMaxDevices = 64;
 struct DeviceInfo {
   int sms = 0;
   bool attrs_done = false;
+  // wisp_verify_step runs the acceptance row statistics on `side`, forked from and joined back
+  // into the caller's stream with these events; step_mu keeps the fork / join of two calls apart
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  std::mutex step_mu;
 };
 DeviceInfo g_dev[kMaxDevices];
 std::mutex g_mu;
@@ -44,6 +49,9 @@ wisp_status device_setup(int *dev_out, int *sms_out) {
     cudaError_t e = attn_simt_setup();
     if (e == cudaSuccess) e = attn_tc_setup();
     if (e == cudaSuccess) e = accept_setup();
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&d.side, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&d.ev_fork, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&d.ev_join, cudaEventDisableTiming);
     if (e != cudaSuccess) return WISP_ERR_CUDA;
     d.sms = sms;
     d.attrs_done = true;
@@ -71,9 +79,20 @@ wisp_status check_attn(const wisp_attn_args *a) {
   return WISP_OK;
 }
 
-int accept_tiles(const wisp_accept_args *c) {
+// Vocabulary slices per logit row for the row-statistics kernel (one warp each): enough warps to
+// keep every SM streaming (48 per SM), slices of at least 256 vectors (4 KB), at most kMaxSlices.
+void accept_slices(const wisp_accept_args *c, int sms, int *slices, int *vps) {
   const int E = c->logits_dtype == WISP_BF16 ? 8 : 4;
-  return (c->V + 32 * E - 1) / (32 * E);
+  const int64_t nvec = ((int64_t)c->V + E - 1) / E;
+  const int64_t rows = c->total_q_rows > 0 ? c->total_q_rows : 1;
+  int64_t S = ((int64_t)48 * sms + rows - 1) / rows;
+  const int64_t by_size = (nvec + 255) / 256;
+  if (S > by_size) S = by_size;
+  if (S > kMaxSlices) S = kMaxSlices;
+  if (S < 1) S = 1;
+  const int64_t v = ((nvec + S - 1) / S + 31) / 32 * 32;
+  *vps = (int)v;
+  *slices = (int)((nvec + v - 1) / v);
 }
 
 wisp_status check_accept(const wisp_accept_args *c) {
@@ -88,6 +107,7 @@ wisp_status check_accept(const wisp_accept_args *c) {
     return WISP_ERR_INVALID_ARG;
   if (c->V > (1 << 24)) return WISP_ERR_UNSUPPORTED;  // vocabulary limit of the acceptance kernel
   if ((int64_t)c->B * 8 > INT32_MAX) return WISP_ERR_UNSUPPORTED;
+  if ((int64_t)c->total_q_rows * kMaxSlices > INT32_MAX) return WISP_ERR_UNSUPPORTED;
   return WISP_OK;
 }
 
@@ -115,6 +135,11 @@ Layout make_layout(const wisp_attn_args *a, const wisp_accept_args *c, int sms) 
     L.items = take(sizeof(WorkItem) * (size_t)L.max_items);
     L.order = take(sizeof(int32_t) * (size_t)L.max_items);
     L.partials = take(sizeof(float) * (size_t)L.partial_cap);
+  }
+  if (c && c->B > 0) {
+    int S = 1, vps = 0;
+    accept_slices(c, sms, &S, &vps);
+    L.row_parts = take(sizeof(RowPart) * (size_t)c->total_q_rows * S);
   }
   L.total = off;
   return L;
@@ -201,7 +226,7 @@ wisp_status launch_attention(const wisp_attn_args *a, void *ws, const Layout &L,
   return attn_combine_launch(ap, bf, s) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
 }
 
-wisp_status launch_accept(const wisp_accept_args *c, void *ws, const Layout &L, int sms, cudaStream_t s) {
+AcceptParams accept_params(const wisp_accept_args *c, void *ws, const Layout &L, int sms) {
   AcceptParams ap;
   std::memset(&ap, 0, sizeof ap);
   ap.B = c->B;
@@ -210,6 +235,9 @@ wisp_status launch_accept(const wisp_accept_args *c, void *ws, const Layout &L, 
   const size_t esz = bf ? 2 : 4;
   ap.vec_z = ((uintptr_t)c->target_logits % 16 == 0) && ((size_t)c->V * esz % 16 == 0);
   ap.vec_q = c->draft_probs && ((uintptr_t)c->draft_probs % 16 == 0) && ((size_t)c->V * 4 % 16 == 0);
+  accept_slices(c, sms, &ap.slices, &ap.vps);
+  ap.total_rows = c->total_q_rows;
+  ap.parts = at<RowPart>(ws, L.row_parts);
   ap.request_ids = c->request_ids;
   ap.draft_lens = c->draft_lens;
   ap.logits = c->target_logits;
@@ -234,8 +262,14 @@ wisp_status launch_accept(const wisp_accept_args *c, void *ws, const Layout &L, 
   if (C > max_c) C = max_c;
   ap.cluster = (int)C;
   ap.vpc = (int)(((nvec + C - 1) / C + 31) / 32 * 32);
-  ap.prefetch = c->B < sms ? 1 : 0;
-  const cudaError_t e = accept_launch(ap, bf, s);
+  return ap;
+}
+
+wisp_status launch_accept(const wisp_accept_args *c, void *ws, const Layout &L, int sms, cudaStream_t s) {
+  const AcceptParams ap = accept_params(c, ws, L, sms);
+  const bool bf = c->logits_dtype == WISP_BF16;
+  cudaError_t e = accept_stats_launch(ap, bf, s);
+  if (e == cudaSuccess) e = accept_walk_launch(ap, bf, s);
   return e == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
 }
 
@@ -251,9 +285,11 @@ wisp_status launch_plan(const wisp_attn_args *a, const wisp_accept_args *c, void
 }  // namespace
 
 // Workspace of wisp_verify_accept_noalloc: status word, per-request offsets and flags, planner
-// header.  128 KiB holds them for batches of up to kNoAllocMaxBatch requests.
-constexpr size_t kNoAllocScratchBytes = 128 << 10;
+// header and the statistics of every logit row.  4 MiB holds them for batches of up to
+// kNoAllocMaxBatch requests and kNoAllocMaxRows logit rows.
+constexpr size_t kNoAllocScratchBytes = 4 << 20;
 constexpr int kNoAllocMaxBatch = 8192;
+constexpr int kNoAllocMaxRows = 131072;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 namespace {
@@ -323,10 +359,24 @@ wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args 
   const Layout L = make_layout(attn, acc, sms);
   if ((st = check_ws(ws, ws_bytes, L)) != WISP_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if ((st = launch_plan(attn, acc, ws, L, s)) != WISP_OK) return st;
-  if (attn->B == 0) return WISP_OK;
-  if ((st = launch_attention(attn, ws, L, s)) != WISP_OK) return st;
-  return launch_accept(acc, ws, L, sms, s);
+  if (attn->B == 0) return launch_plan(attn, acc, ws, L, s);
+  // The row statistics of the acceptance pass read only the logits, so they run on the library's
+  // side stream while the planner (one CTA) runs on `s`; the walk and draw follow the attention
+  // on `s` once the statistics are joined back.  (Running the walk concurrently with the
+  // attention was measured to gain nothing: both are issue-bound while active.)
+  DeviceInfo &d = g_dev[dev];
+  std::lock_guard<std::mutex> lk(d.step_mu);
+  const AcceptParams ap = accept_params(acc, ws, L, sms);
+  const bool bf = acc->logits_dtype == WISP_BF16;
+  bool ok = cudaEventRecord(d.ev_fork, s) == cudaSuccess && cudaStreamWaitEvent(d.side, d.ev_fork, 0) == cudaSuccess;
+  ok = ok && accept_stats_launch(ap, bf, d.side) == cudaSuccess;
+  // join what was forked even after a failed launch, so that `s` never runs ahead of `side`
+  const bool joined = cudaEventRecord(d.ev_join, d.side) == cudaSuccess;
+  ok = ok && launch_plan(attn, acc, ws, L, s) == WISP_OK;
+  ok = ok && launch_attention(attn, ws, L, s) == WISP_OK;
+  const bool waited = joined && cudaStreamWaitEvent(s, d.ev_join, 0) == cudaSuccess;
+  ok = ok && waited && accept_walk_launch(ap, bf, s) == cudaSuccess;
+  return ok && waited ? WISP_OK : WISP_ERR_CUDA;
 }
 
 wisp_status wisp_verify_get_device_status(const void *ws, int32_t *code, int64_t *request_id) {
@@ -349,7 +399,7 @@ wisp_status wisp_verify_get_device_status(const void *ws, int32_t *code, int64_t
 wisp_status wisp_verify_accept_noalloc(const wisp_accept_args *acc, void *stream) {
   wisp_status st = check_accept(acc);
   if (st != WISP_OK) return st;
-  if (acc->B > kNoAllocMaxBatch) return WISP_ERR_UNSUPPORTED;  // beyond the fixed scratch
+  if (acc->B > kNoAllocMaxBatch || acc->total_q_rows > kNoAllocMaxRows) return WISP_ERR_UNSUPPORTED;
   int dev = 0, sms = 0;
   if ((st = device_setup(&dev, &sms)) != WISP_OK) return st;
   const Layout L = make_layout(nullptr, acc, sms);

@@ -54,7 +54,7 @@ struct Cfg {
   static constexpr int HALVES = D / 64;
   static constexpr int Q_BYTES = kM * D * 2;
   static constexpr int KV_TILE = kBN * D * 2;  // K (or V) of one tile
-  static constexpr int NSTAGE = D == 128 ? 4 : 6;
+  static constexpr int NSTAGE = D == 128 ? 3 : 6;
   static constexpr int P_BYTES = kM * kBN * 2;
   static constexpr int RING = 4;               // slots of the item ring
   static constexpr int OFF_Q = 0;
@@ -804,6 +804,10 @@ cudaError_t attn_tc_setup() {
     e = cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<128>::SMEM);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<64>::SMEM);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
   return e;
 }
 

@@ -28,6 +28,17 @@ __device__ __forceinline__ void report(DeviceStatus *st, int32_t code, const int
 constexpr int kMaxRowsPerHead = 128;  // (Hq/Hkv) * (k+1) rows per KV head per work item
 constexpr int kMaxDraft = 1024;       // k_r limit of the acceptance kernels
 
+// Hardware 2^x (ex2.approx.ftz.f32).  Over every float x in [-126, 0] its relative error is below
+// 2^-22.7 (measured exhaustively on GB300 by tests/test_ex2_bound_gpu.py); the acceptance kernels'
+// certified bounds use kEx2RelErr for it.  Below -126 the result flushes to zero.
+constexpr float kEx2RelErr = 0x1p-22f;
+constexpr float kLog2e = 1.4426950408889634f;  // log2(e) rounded to float
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // Per-request flags written by the planner
 enum : int32_t { REQ_OK = 0, REQ_BAD = 1 };
 

@@ -39,6 +39,7 @@ struct Layout {
   size_t items = 0;           // WorkItem [max_items]
   size_t order = 0;           // int32 [max_items]  dispatch order of the items (largest first)
   size_t partials = 0;        // float [partial_cap]
+  size_t row_parts = 0;       // RowPart [total_q_rows, slices] statistics of the logit rows
   size_t total = 0;
   int64_t max_items = 0;
   int64_t partial_cap = 0;    // floats

@@ -96,15 +96,16 @@ def test_accept_rejects_bad_arguments(lib, kw):
     assert rc in (wb.WISP_ERR_INVALID_ARG, wb.WISP_ERR_UNSUPPORTED)
 
 
-@pytest.mark.parametrize("kw", BAD_ACC + [dict(B=8193, total_q_rows=8193, total_draft=0)],
-                         ids=[str(k) for k in BAD_ACC] + ["B=8193"])
+@pytest.mark.parametrize("kw", BAD_ACC + [dict(B=8193, total_q_rows=8193, total_draft=0),
+                                           dict(B=100, total_q_rows=131073, total_draft=0)],
+                         ids=[str(k) for k in BAD_ACC] + ["B=8193", "rows=131073"])
 def test_accept_noalloc_rejects_bad_arguments(lib, kw):
     # checked on the host before any device call; a batch beyond the fixed scratch is unsupported
     from paper_2601_11652_gb300 import binding as wb
     c = _acc(**kw)
     rc = lib.wisp_verify_accept_noalloc(ctypes.byref(c), None)
     assert rc in (wb.WISP_ERR_INVALID_ARG, wb.WISP_ERR_UNSUPPORTED)
-    if kw.get("B") == 8193:
+    if kw.get("B") == 8193 or kw.get("total_q_rows") == 131073:
         assert rc == wb.WISP_ERR_UNSUPPORTED
 
 
