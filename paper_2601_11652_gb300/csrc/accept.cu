@@ -24,6 +24,7 @@
 // elements.
 #include <cooperative_groups.h>
 #include <cstring>
+#include <type_traits>
 
 #include "accept.cuh"
 
@@ -106,11 +107,55 @@ __device__ __forceinline__ void load_q(const float *qrow, int64_t v0, int V, boo
   }
 }
 
+// bf16 logits take few distinct values, so the draw looks exp(u - m) up in a table of the bf16
+// values u in the table's range, computed once per CTA with the very same double-float function
+// (the results are bit-identical to computing every element); other values are computed directly.
+__device__ __forceinline__ int exp_tab_index(uint32_t bits16) {
+  const uint32_t d = ((bits16 >> 7) & 0xFFu) - (uint32_t)kExpTabLo;  // wraps below the range
+  if (d >= (uint32_t)kExpTabBinades) return -1;
+  return (int)((((bits16 >> 15) * kExpTabBinades + d) << 7) | (bits16 & 0x7Fu));
+}
+__device__ __forceinline__ uint32_t exp_tab_bits(int idx) {
+  const uint32_t sign = (uint32_t)idx / (kExpTabBinades * 128), rem = (uint32_t)idx % (kExpTabBinades * 128);
+  return (sign << 15) | (((rem >> 7) + kExpTabLo) << 7) | (rem & 0x7Fu);
+}
+
 // Double-float weight of one element in the draw: exp(z - m) [- q * Z, clamped at 0].
 __device__ __forceinline__ ff draw_weight(float z, float m, bool residual, float q, ff Zff, const float *th,
                                           const float *tl) {
   const ff x = ff_two_sum(z, -m);
   ff e = ff_exp_nonpos(x.hi, x.lo, th, tl);
+  if (residual) {
+    e = ff_add(e, ff_neg(ff_mul_f(Zff, q)));
+    if (!(e.hi > 0.0f)) e = {0.0f, 0.0f};
+  }
+  return e;
+}
+
+// Out-of-table values (rare for logits): the direct double-float exp, kept out of line so that the
+// unrolled loops stay small.
+__device__ __noinline__ ff exp_direct(float z, float m, const float *th, const float *tl) {
+  return draw_weight(z, m, false, 0.0f, ff{}, th, tl);
+}
+
+// exp(z - m) of element i of vector w; bf16: from the table when z is in its range.
+template <typename LT>
+__device__ __forceinline__ ff elem_exp(const uint4 &w, int i, float m, const ff *tab, const float *th, const float *tl);
+template <>
+__device__ __forceinline__ ff elem_exp<float>(const uint4 &w, int i, float m, const ff *, const float *th, const float *tl) {
+  return draw_weight(vec_elem<float>(w, i), m, false, 0.0f, ff{}, th, tl);
+}
+template <>
+__device__ __forceinline__ ff elem_exp<uint16_t>(const uint4 &w, int i, float m, const ff *tab, const float *th,
+                                                 const float *tl) {
+  const uint32_t u = (i >> 1) == 0 ? w.x : (i >> 1) == 1 ? w.y : (i >> 1) == 2 ? w.z : w.w;
+  const int idx = exp_tab_index((i & 1) ? (u >> 16) : (u & 0xFFFFu));
+  if (idx >= 0) return tab[idx];
+  return exp_direct(vec_elem<uint16_t>(w, i), m, th, tl);
+}
+
+// Draw weight from e = exp(z - m): e itself, or the residual max(0, e - q Z) (as draw_weight).
+__device__ __forceinline__ ff weight_from(ff e, bool residual, float q, ff Zff) {
   if (residual) {
     e = ff_add(e, ff_neg(ff_mul_f(Zff, q)));
     if (!(e.hi > 0.0f)) e = {0.0f, 0.0f};
@@ -303,7 +348,7 @@ __global__ void __launch_bounds__(NT) row_stats_kernel(const __grid_constant__ A
 template <typename LT>
 __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ AcceptParams p) {
   constexpr int E = LTraits<LT>::E;
-  extern __shared__ ff s_tile[];  // [rounds * NW] per-(round, warp) draw sums
+  extern __shared__ ff s_tile[];  // [rounds * NW] per-(round, warp) draw sums, then the exp table (bf16)
   __shared__ float s_th[256], s_tl[256];
   __shared__ RowStats s_wst[NW];
   __shared__ RowStats s_pub[2];   // this CTA's published totals (ring of 2)
@@ -511,7 +556,24 @@ __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ Acce
   const LT *row = logits + (Q0 + L) * (int64_t)V;
   const float *qrow = p.draft_probs + (D0 + L) * (int64_t)V;
   bool residual = L < k;
-  if (residual && !have_Zff) Zff = row_Zff(row, m);
+  // exp(u - m) of row L for the bf16 values u of the table's range
+  ff *s_etab = s_tile + rounds * NW;
+  if (std::is_same<LT, uint16_t>::value) {
+    for (int idx = tid; idx < kExpTabSize; idx += NT) {
+      const float u = bf16_bits_to_float(exp_tab_bits(idx));
+      s_etab[idx] = u > m ? ff{0.0f, 0.0f} : draw_weight(u, m, false, 0.0f, ff{}, s_th, s_tl);  // u > m never occurs
+    }
+    __syncthreads();
+  }
+  if (residual && !have_Zff) {
+    ff acc = {0.0f, 0.0f};
+    for (int64_t vi = vlo + tid; vi < vhi; vi += NT) {
+      const uint4 w = load_vec<LT>(row, vi, V, vec_z);
+#pragma unroll
+      for (int i = 0; i < E; ++i) acc = ff_add(acc, elem_exp<LT>(w, i, m, s_etab, s_th, s_tl));
+    }
+    Zff = cluster_total(acc);
+  }
   ff S = {0.0f, 0.0f};
   for (;;) {
     ff run = {0.0f, 0.0f};
@@ -529,7 +591,7 @@ __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ Acce
         }
 #pragma unroll
         for (int i = 0; i < E; ++i)
-          part = ff_add(part, draw_weight(vec_elem<LT>(w, i), m, residual, q[i], Zff, s_th, s_tl));
+          part = ff_add(part, weight_from(elem_exp<LT>(w, i, m, s_etab, s_th, s_tl), residual, q[i], Zff));
       }
       for (int o = 16; o > 0; o >>= 1) part = ff_add(part, ff_shfl_xor(part, o));
       if (lane == 0) s_tile[rd * NW + warp] = part;
@@ -622,7 +684,7 @@ __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ Acce
         }
 #pragma unroll
         for (int i = 0; i < E; ++i) {
-          wts[i] = draw_weight(vec_elem<LT>(w, i), m, residual, q[i], Zff, s_th, s_tl);
+          wts[i] = weight_from(elem_exp<LT>(w, i, m, s_etab, s_th, s_tl), residual, q[i], Zff);
           lsum = ff_add(lsum, wts[i]);
         }
       }
@@ -699,7 +761,7 @@ cudaError_t walk_t(const AcceptParams &ap, cudaStream_t s) {
   memset(&cfg, 0, sizeof cfg);
   cfg.gridDim = dim3((unsigned)((int64_t)ap.B * ap.cluster));
   cfg.blockDim = dim3(NT);
-  cfg.dynamicSmemBytes = (size_t)rounds * NW * sizeof(ff);
+  cfg.dynamicSmemBytes = (size_t)rounds * NW * sizeof(ff) + (std::is_same<LT, uint16_t>::value ? kExpTabSize * sizeof(ff) : 0);
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;

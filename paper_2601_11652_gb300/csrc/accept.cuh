@@ -8,6 +8,11 @@ namespace wisp {
 constexpr int kAcceptThreads = 256;  // 8 warps per CTA
 constexpr int kMaxAcceptCluster = 8;
 constexpr int kPreload = 256;        // decision inputs gathered up front for the first rows
+// Per-CTA table of exp(u - m) for the bf16 values u with 2^-8 <= |u| < 2^6 (exponent fields
+// kExpTabLo .. kExpTabLo + kExpTabBinades - 1, both signs), used by the draw.
+constexpr int kExpTabLo = 119;
+constexpr int kExpTabBinades = 14;
+constexpr int kExpTabSize = 2 * kExpTabBinades * 128;
 
 // Statistics of one vocabulary slice of one logit row (written by row_stats_kernel): running max,
 // double-float sum of exp(z - m), the error terms of the certified bound, rescale count.
