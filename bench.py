@@ -227,6 +227,21 @@ def _time_loop(fn, steps, flush, torch):
     return [s.elapsed_time(e) for s, e in zip(starts, ends)]
 
 
+def aggregate_ranks(total_ms: float, verified: int, world: int, device):
+    """Whole-job numbers of N replicas: the slowest rank's time (max) and every rank's verified
+    tokens (sum).  The replicas verify independent batches, so this is the only collective."""
+    if world <= 1:
+        return total_ms, verified
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([total_ms], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    v = torch.tensor([verified], device=device, dtype=torch.int64)
+    dist.all_reduce(v, op=dist.ReduceOp.SUM)
+    dist.barrier()
+    return float(t.item()), int(v.item())
+
+
 def run_ours(args, batch, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -266,16 +281,7 @@ def run_ours(args, batch, rank, world, local_rank):
     code, rid = db.device_status()
     if code != 0:
         raise RuntimeError(f"device status {code} at request {rid} after the timed steps")
-    total_ms = sum(ms)
-    verified_all = verified
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-        v = torch.tensor([verified], device=dev, dtype=torch.int64)
-        dist.all_reduce(v, op=dist.ReduceOp.SUM)
-        verified_all = int(v.item())
-        dist.barrier()
+    total_ms, verified_all = aggregate_ranks(sum(ms), verified, world, dev)
     ms_per_step = total_ms / args.steps
     value = verified_all / (ms_per_step / 1e3)
 
@@ -342,6 +348,61 @@ def _e2e(db, batch, args, flush, torch, verified):
             "note": "the paged KV cache (prefix cache) stays resident in HBM; every other input is copied in"}
 
 
+# --------------------------------------------------------------------------
+# latency table for the verification-time estimator (Sec. 4.4, Eq. batch_time)
+# --------------------------------------------------------------------------
+LT_BATCHES = (1, 2, 4, 8, 16, 32, 64, 128, 256, 512)
+LT_DRAFTS = (1, 2, 4, 8, 16)   # draft tokens per request (sum k = B * this)
+
+
+def latency_table(path: str, max_b: int, reps: int):
+    """Step / attention / acceptance times over batch size x draft length on the Llama-3-8B-shaped
+    layer (32/8/128 bf16 KV, V = 128256, contexts ~ U{512..4096}), with the estimator's features;
+    writes a CSV and fits T_step = a N_linear + b_compute N_interactions + b_read N_cached + c."""
+    import csv
+    import torch
+    from paper_2601_11652_gb300 import build, estimator as est, workload as wl
+    from paper_2601_11652_gb300.device_batch import DeviceBatch
+    build.build()
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    rng = np.random.default_rng(2601_11652)
+    rows = []
+    for B in LT_BATCHES:
+        if B > max_b:
+            continue
+        for kk in LT_DRAFTS:
+            k = np.full(B, kk, np.int32)
+            c = rng.integers(512, 4097, size=B).astype(np.int32)
+            batch = wl.make_batch_from_lengths(f"lt_b{B}_k{kk}", draft_lens=k, context_lens=c, Hq=32, Hkv=8, D=128,
+                                               V=128256, dtype="bf16", sigma=float(wl.sigma_for_alpha(0.7)),
+                                               key=(7000 + B, kk), shuffle_blocks=False, extra_blocks=1)
+            db = DeviceBatch.from_host(batch)
+            for _ in range(3):
+                db.step()
+            t = {}
+            for fn in ("step", "attention", "accept"):
+                ms = _time_loop(getattr(db, fn), reps, flush, torch)
+                t[fn] = float(np.median(ms))
+            code, rid = db.device_status()
+            if code != 0:
+                raise RuntimeError(f"device status {code} at request {rid}")
+            f = est.features(c, k)
+            rows.append({"B": B, "k": kk, "sum_k": int(k.sum()), "N_linear": f[0], "N_interactions": f[1],
+                         "N_cached": f[2], "t_step_ms": t["step"], "t_attention_ms": t["attention"],
+                         "t_accept_ms": t["accept"]})
+            print(json.dumps(rows[-1]), flush=True)
+            del db
+            torch.cuda.empty_cache()
+    with open(path, "w", newline="") as fh:
+        w = csv.DictWriter(fh, fieldnames=list(rows[0]))
+        w.writeheader()
+        w.writerows(rows)
+    X = np.array([[r[n] for n in est.FEATURES] for r in rows])
+    y = np.array([r["t_step_ms"] for r in rows]) * 1e-3
+    fit = est.fit_with_validation(X, y)
+    print(fit.report("s"), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -349,7 +410,14 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--workload", default="llama3_8b_b32")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--latency-table", metavar="CSV", help="sweep batch size x draft length for the estimator "
+                    "(Sec. 4.4) instead of the benchmark line; writes CSV and prints the fit")
+    ap.add_argument("--lt-max-b", type=int, default=512)
+    ap.add_argument("--lt-reps", type=int, default=20)
     args = ap.parse_args()
+    if args.latency_table:
+        latency_table(args.latency_table, args.lt_max_b, args.lt_reps)
+        return
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", 1))
     local_rank = int(os.environ.get("LOCAL_RANK", 0))

@@ -150,7 +150,7 @@ __device__ __forceinline__ ff elem_exp<uint16_t>(const uint4 &w, int i, float m,
                                                  const float *tl) {
   const uint32_t u = (i >> 1) == 0 ? w.x : (i >> 1) == 1 ? w.y : (i >> 1) == 2 ? w.z : w.w;
   const int idx = exp_tab_index((i & 1) ? (u >> 16) : (u & 0xFFFFu));
-  if (idx >= 0) return tab[idx];
+  if (tab && idx >= 0) return tab[idx];
   return exp_direct(vec_elem<uint16_t>(w, i), m, th, tl);
 }
 
@@ -557,8 +557,9 @@ __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ Acce
   const float *qrow = p.draft_probs + (D0 + L) * (int64_t)V;
   bool residual = L < k;
   // exp(u - m) of row L for the bf16 values u of the table's range
-  ff *s_etab = s_tile + rounds * NW;
-  if (std::is_same<LT, uint16_t>::value) {
+  // (only for rows much longer than the table)
+  ff *s_etab = std::is_same<LT, uint16_t>::value && V >= kExpTabMinV ? s_tile + rounds * NW : nullptr;
+  if (s_etab) {
     for (int idx = tid; idx < kExpTabSize; idx += NT) {
       const float u = bf16_bits_to_float(exp_tab_bits(idx));
       s_etab[idx] = u > m ? ff{0.0f, 0.0f} : draw_weight(u, m, false, 0.0f, ff{}, s_th, s_tl);  // u > m never occurs
@@ -761,7 +762,8 @@ cudaError_t walk_t(const AcceptParams &ap, cudaStream_t s) {
   memset(&cfg, 0, sizeof cfg);
   cfg.gridDim = dim3((unsigned)((int64_t)ap.B * ap.cluster));
   cfg.blockDim = dim3(NT);
-  cfg.dynamicSmemBytes = (size_t)rounds * NW * sizeof(ff) + (std::is_same<LT, uint16_t>::value ? kExpTabSize * sizeof(ff) : 0);
+  const bool tab = std::is_same<LT, uint16_t>::value && ap.V >= kExpTabMinV;
+  cfg.dynamicSmemBytes = (size_t)rounds * NW * sizeof(ff) + (tab ? kExpTabSize * sizeof(ff) : 0);
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;

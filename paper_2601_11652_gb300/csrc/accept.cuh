@@ -13,6 +13,7 @@ constexpr int kPreload = 256;        // decision inputs gathered up front for th
 constexpr int kExpTabLo = 119;
 constexpr int kExpTabBinades = 14;
 constexpr int kExpTabSize = 2 * kExpTabBinades * 128;
+constexpr int kExpTabMinV = 16384;  // vocabularies smaller than this compute every exp directly
 
 // Statistics of one vocabulary slice of one logit row (written by row_stats_kernel): running max,
 // double-float sum of exp(z - m), the error terms of the certified bound, rescale count.

@@ -28,6 +28,7 @@ from __future__ import annotations
 
 import dataclasses
 import math
+import os
 from concurrent.futures import ThreadPoolExecutor
 
 import numpy as np
@@ -251,27 +252,30 @@ def make_batch_from_lengths(name, *, draft_lens, context_lens, Hq, Hkv, D, V, dt
     qs = np.concatenate([[0], np.cumsum(draft_lens + 1)])
     ds = np.concatenate([[0], np.cumsum(draft_lens)])
     z_f32 = (lambda rows: bf16_bits_to_f32(logits[rows])) if dtype == "bf16" else (lambda rows: logits[rows])
-    noise_rng = _rng(*key, 6)
-    tok_rng = _rng(*key, 7)
-    for r in range(B):
+    def one_request(r):
+        # request r's noise and token draws come from its own stream, so requests run in parallel
         k = int(draft_lens[r])
         if k == 0:
-            continue
+            return
+        rng = _rng(*key, 6, r)
         base = z_f32(np.arange(qs[r], qs[r] + k)).astype(np.float64)
-        x = base + sigma[r] * noise_rng.standard_normal((k, V))
+        x = base + sigma[r] * rng.standard_normal((k, V))
         x -= x.max(axis=1, keepdims=True)
         np.exp(x, out=x)
         x /= x.sum(axis=1, keepdims=True)
         qf = x.astype(np.float32)
         draft_probs[ds[r]: ds[r] + k] = qf
         cdf = np.cumsum(qf.astype(np.float64), axis=1)
-        u = tok_rng.random(k)
+        u = rng.random(k)
         for j in range(k):
             t = int(np.searchsorted(cdf[j], u[j] * cdf[j, -1], side="right"))
             t = min(t, V - 1)
             while qf[j, t] == 0.0 and t > 0:  # never hand out a token the draft gave zero mass
                 t -= 1
             draft_tokens[ds[r] + j] = t
+
+    with ThreadPoolExecutor(max_workers=min(32, os.cpu_count() or 1)) as ex:
+        list(ex.map(one_request, range(B)))
     accept_u = _rng(*key, 8).random(T_d, dtype=np.float32)
     sample_u = _rng(*key, 9).random(B, dtype=np.float32)
     return VerifyBatch(
