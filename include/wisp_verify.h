@@ -78,7 +78,8 @@ typedef enum {
   WISP_DEV_BAD_PROB = 4,     /* a draft probability q(y) that is negative or NaN, or a logit row
                                 with no finite maximum / non-finite normaliser */
   WISP_DEV_UNSUPPORTED = 5,  /* (Hq / Hkv) * (k_r + 1) > 128 query rows, or k_r > 1024 */
-  WISP_DEV_TIMEOUT = 6       /* a bounded device-side wait gave up (no kernel waits unboundedly) */
+  WISP_DEV_TIMEOUT = 6,      /* a bounded device-side wait gave up (no kernel waits unboundedly) */
+  WISP_DEV_NO_BLOCKS = 7     /* (wisp_kv.h) the free page pool could not serve the request */
 } wisp_device_code;
 
 typedef enum { WISP_F32 = 0, WISP_BF16 = 1 } wisp_dtype;

@@ -38,6 +38,14 @@ class wisp_accept_args(ctypes.Structure):
                 ("sample_uniforms", _P), ("accepted_len", _P), ("next_token", _P)]
 
 
+class wisp_kv_args(ctypes.Structure):
+    _fields_ = [("B", _I32), ("Hkv", _I32), ("D", _I32), ("block_size", _I32), ("max_blocks_per_seq", _I32),
+                ("num_blocks", _I32), ("total_q_rows", _I32), ("request_ids", _P), ("draft_lens", _P),
+                ("context_lens", _P), ("block_tables", _P), ("free_blocks", _P), ("free_count", _P),
+                ("kv_dtype", ctypes.c_int), ("k_cache", _P), ("v_cache", _P), ("k_new", _P), ("v_new", _P),
+                ("accepted_len", _P)]
+
+
 class WispError(RuntimeError):
     def __init__(self, fn: str, code: int, text: str):
         super().__init__(f"{fn}: {text} (status {code})")
@@ -47,7 +55,8 @@ class WispError(RuntimeError):
 _lib = None
 
 EXPORTED = ["wisp_verify_workspace_size", "wisp_verify_attention", "wisp_verify_accept", "wisp_verify_step",
-            "wisp_verify_get_device_status", "wisp_verify_status_string", "wisp_verify_device_code_string"]
+            "wisp_verify_get_device_status", "wisp_verify_status_string", "wisp_verify_device_code_string",
+            "wisp_verify_accept_noalloc", "wisp_kv_workspace_size", "wisp_kv_reserve_append", "wisp_kv_commit"]
 
 
 def lib_path() -> str:
@@ -81,6 +90,12 @@ def load(path: str | None = None):
     lib.wisp_verify_status_string.restype = ctypes.c_char_p
     lib.wisp_verify_device_code_string.argtypes = [_I32]
     lib.wisp_verify_device_code_string.restype = ctypes.c_char_p
+    KP = ctypes.POINTER(wisp_kv_args)
+    lib.wisp_kv_workspace_size.argtypes = [KP]
+    lib.wisp_kv_workspace_size.restype = ctypes.c_size_t
+    for fn in ("wisp_kv_reserve_append", "wisp_kv_commit"):
+        getattr(lib, fn).argtypes = [KP, _P, ctypes.c_size_t, _P]
+        getattr(lib, fn).restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -192,3 +207,40 @@ def wisp_verify_get_device_status(workspace: torch.Tensor) -> tuple[int, int]:
     _check("wisp_verify_get_device_status",
            load().wisp_verify_get_device_status(_ptr(workspace), ctypes.byref(code), ctypes.byref(rid)))
     return int(code.value), int(rid.value)
+
+
+# ---- paged KV maintenance (include/wisp_kv.h) ---------------------------------------------------
+def make_kv_args(*, draft_lens, context_lens, block_tables, free_blocks, free_count, k_cache=None, v_cache=None,
+                 k_new=None, v_new=None, accepted_len=None, request_ids=None, total_q_rows=None) -> wisp_kv_args:
+    """Fill wisp_kv_args from device tensors (k_cache / v_cache [num_blocks, Hkv, 16, D])."""
+    a = wisp_kv_args()
+    a.B = draft_lens.shape[0]
+    a.max_blocks_per_seq = block_tables.shape[1]
+    a.num_blocks = free_blocks.shape[0]
+    ref = k_cache if k_cache is not None else k_new
+    a.Hkv = ref.shape[1] if ref is not None else 1
+    a.D = ref.shape[-1] if ref is not None else 128
+    a.block_size = 16
+    a.total_q_rows = int(draft_lens.sum().item()) + a.B if total_q_rows is None else total_q_rows
+    a.request_ids, a.draft_lens, a.context_lens = _ptr(request_ids), _ptr(draft_lens), _ptr(context_lens)
+    a.block_tables, a.free_blocks, a.free_count = _ptr(block_tables), _ptr(free_blocks), _ptr(free_count)
+    a.kv_dtype = _dtype_code(ref) if ref is not None else WISP_BF16
+    a.k_cache, a.v_cache, a.k_new, a.v_new = _ptr(k_cache), _ptr(v_cache), _ptr(k_new), _ptr(v_new)
+    a.accepted_len = _ptr(accepted_len)
+    return a
+
+
+def wisp_kv_workspace_size(kv: wisp_kv_args) -> int:
+    n = load().wisp_kv_workspace_size(ctypes.byref(kv))
+    if n == 0:
+        raise WispError("wisp_kv_workspace_size", WISP_ERR_INVALID_ARG, "invalid arguments")
+    return int(n)
+
+
+def wisp_kv_reserve_append(kv: wisp_kv_args, workspace: torch.Tensor, stream=None) -> None:
+    _check("wisp_kv_reserve_append", load().wisp_kv_reserve_append(
+        ctypes.byref(kv), _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def wisp_kv_commit(kv: wisp_kv_args, workspace: torch.Tensor, stream=None) -> None:
+    _check("wisp_kv_commit", load().wisp_kv_commit(ctypes.byref(kv), _ptr(workspace), workspace.numel(), _stream(stream)))

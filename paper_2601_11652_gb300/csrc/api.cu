@@ -433,6 +433,7 @@ const char *wisp_verify_device_code_string(int32_t code) {
     case WISP_DEV_BAD_PROB: return "bad probability or logit row";
     case WISP_DEV_UNSUPPORTED: return "unsupported request shape";
     case WISP_DEV_TIMEOUT: return "device wait timed out";
+    case WISP_DEV_NO_BLOCKS: return "no free KV pages";
   }
   return "unknown device code";
 }

@@ -21,7 +21,7 @@ struct DeviceStatus {
 // Record the first device-side error; later errors are dropped.
 __device__ __forceinline__ void report(DeviceStatus *st, int32_t code, const int64_t *request_ids, int r) {
   if (atomicCAS(&st->code, 0, code) == 0) {
-    st->request_id = request_ids ? request_ids[r] : (int64_t)r;
+    st->request_id = request_ids && r >= 0 ? request_ids[r] : (int64_t)r;  // r < 0: not one request
   }
 }
 

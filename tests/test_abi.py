@@ -9,6 +9,7 @@ import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 HEADER = os.path.join(ROOT, "include", "wisp_verify.h")
+HEADERS = [HEADER, os.path.join(ROOT, "include", "wisp_kv.h")]
 
 
 @pytest.fixture(scope="module")
@@ -19,9 +20,11 @@ def lib():
 
 
 def declared_functions():
-    text = open(HEADER).read()
-    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(wisp_verify_\w+)\s*\(", text)))
+    names = set()
+    for h in HEADERS:
+        text = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        names |= set(re.findall(r"\b(wisp_(?:verify|kv)_\w+)\s*\(", text))
+    return sorted(names)
 
 
 def test_header_declares_the_abi():
@@ -43,7 +46,8 @@ def test_library_exports_every_declared_symbol(lib):
 
 def test_header_compiles_as_c(tmp_path):
     src = tmp_path / "t.c"
-    src.write_text('#include "wisp_verify.h"\nint main(void){ return (int)sizeof(wisp_attn_args) > 0 ? 0 : 1; }\n')
+    src.write_text('#include "wisp_verify.h"\n#include "wisp_kv.h"\n'
+                   'int main(void){ return (int)(sizeof(wisp_attn_args) + sizeof(wisp_kv_args)) > 0 ? 0 : 1; }\n')
     subprocess.run(["gcc", "-std=c99", "-Wall", "-Werror", "-I", os.path.join(ROOT, "include"), "-c", str(src),
                     "-o", str(tmp_path / "t.o")], check=True)
 
@@ -119,6 +123,6 @@ def test_step_rejects_mismatched_batches(lib):
 def test_status_strings(lib):
     for code in range(5):
         assert lib.wisp_verify_status_string(code)
-    for code in range(7):
-        assert lib.wisp_verify_device_code_string(code)
+    for code in range(8):
+        assert lib.wisp_verify_device_code_string(code) != b"unknown device code"
     assert lib.wisp_verify_get_device_status(None, None, None) == 1
