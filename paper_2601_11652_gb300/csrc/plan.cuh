@@ -22,7 +22,7 @@ struct PlanHeader {
   int32_t pad[4];
 };
 
-constexpr int kItemsPerSM = 4;     // target work items per SM for split-KV
+constexpr int kItemsPerSM = 2;     // target work items per SM for split-KV (measured best of 1, 2, 4, 6, 8)
 constexpr int kMinChunk = 256;     // never split a sequence below this many tokens
 constexpr int kChunkAlign = 128;   // chunk starts are multiples of the KV tile
 
