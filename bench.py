@@ -403,6 +403,39 @@ def latency_table(path: str, max_b: int, reps: int):
     print(fit.report("s"), flush=True)
 
 
+# --------------------------------------------------------------------------
+# verification interference (Sec. 3): solo short, solo long, co-batched
+# --------------------------------------------------------------------------
+def interference(reps: int):
+    """Step time of a short cached request B (500-token prefix, 5 drafts) alone, of a long request A
+    (8 drafts over a growing prefix) alone, and of both in one batch, on the Llama-3-8B-shaped layer:
+    the co-batched step is dictated by A, so B inherits A's latency."""
+    import torch
+    from paper_2601_11652_gb300 import build, workload as wl
+    from paper_2601_11652_gb300.device_batch import DeviceBatch
+    build.build()
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+
+    def t_step(k, c, key):
+        b = wl.make_batch_from_lengths(f"intf{key}", draft_lens=np.array(k, np.int32), context_lens=np.array(c, np.int32),
+                                       Hq=32, Hkv=8, D=128, V=128256, dtype="bf16", sigma=float(wl.sigma_for_alpha(0.7)),
+                                       key=(9100, key), shuffle_blocks=False, extra_blocks=1)
+        db = DeviceBatch.from_host(b)
+        for _ in range(3):
+            db.step()
+        ms = float(np.median(_time_loop(db.step, reps, flush, torch)))
+        del db
+        torch.cuda.empty_cache()
+        return ms
+
+    solo_b = t_step([5], [500], 0)
+    for i, ca in enumerate((1000, 4000, 16000, 64000, 128000)):
+        solo_a = t_step([8], [ca], 1 + i)
+        both = t_step([8, 5], [ca, 500], 10 + i)
+        print(json.dumps({"long_prefix": ca, "solo_short_ms": solo_b, "solo_long_ms": solo_a, "batched_ms": both,
+                          "short_slowdown": both / solo_b}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -414,7 +447,12 @@ def main():
                     "(Sec. 4.4) instead of the benchmark line; writes CSV and prints the fit")
     ap.add_argument("--lt-max-b", type=int, default=512)
     ap.add_argument("--lt-reps", type=int, default=20)
+    ap.add_argument("--interference", action="store_true", help="solo / co-batched step times of a short and a long "
+                    "request (Sec. 3) instead of the benchmark line")
     args = ap.parse_args()
+    if args.interference:
+        interference(20)
+        return
     if args.latency_table:
         latency_table(args.latency_table, args.lt_max_b, args.lt_reps)
         return

@@ -159,6 +159,14 @@ wisp_status wisp_verify_attention(const wisp_attn_args *attn, void *workspace, s
 wisp_status wisp_verify_accept(const wisp_accept_args *acc, void *workspace, size_t workspace_bytes,
                                void *stream);
 
+/* Greedy (temperature 0) variant of the acceptance pass: sampling at temperature 0 takes the most
+ * likely token, so draft token i is accepted iff it is the argmax of logit row i-1 (the lowest token
+ * id among equal maxima), the walk stops at the first mismatch (Eq. 2) and the extra token is the
+ * argmax of row L.  draft_probs, accept_uniforms and sample_uniforms are not read (may be NULL).
+ * NaN logits are never chosen; a row without a finite logit is flagged WISP_DEV_BAD_PROB. */
+wisp_status wisp_verify_accept_greedy(const wisp_accept_args *acc, void *workspace, size_t workspace_bytes,
+                                      void *stream);
+
 /* Enqueue one whole verification step (Sec. 4.5): attention and acceptance.  The two parts
  * read disjoint inputs; draft_lens must describe the same batch in both structs.  Part of the
  * acceptance pass (its row statistics) runs on a stream owned by the library, forked from and

@@ -123,3 +123,44 @@ def row_softmax(row: np.ndarray, dtype: str = "f32") -> np.ndarray:
     p = np.empty(row.shape[-1], dtype=np.float64)
     lib.oracle_row_softmax(row.shape[-1], _dtype_code(dtype), _ptr(row), _ptr(p))
     return p
+
+
+def accept_greedy(batch) -> dict:
+    """Temperature-0 variant of the acceptance rule, written out with numpy (test infrastructure).
+
+    Sampling at temperature 0 takes the most likely token: draft token i is accepted iff it equals
+    the argmax of logit row i-1 (np.argmax: the lowest index among equal maxima), the walk stops at
+    the first mismatch (Eq. 2) and the extra token is the argmax of row L.  NaN logits are never
+    chosen; a row without a finite logit gives status 5 (bad_prob) and L = token = -1.
+    """
+    B = len(batch.draft_lens)
+    V = int(batch.V)
+    if batch.dtype == "bf16":
+        z = (np.asarray(batch.logits, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32)
+    else:
+        z = np.asarray(batch.logits, dtype=np.float32)
+    z = z.reshape(-1, V).astype(np.float64)
+    z = np.where(np.isnan(z), -np.inf, z)
+    L = np.empty(B, np.int32)
+    tok = np.empty(B, np.int32)
+    st = np.zeros(B, np.int32)
+    row0 = 0
+    d0 = 0
+    for r in range(B):
+        k = int(batch.draft_lens[r])
+        L[r], tok[r] = k, -1
+        for i in range(k + 1):
+            row = z[row0 + i]
+            if not np.isfinite(row.max()):
+                st[r], L[r], tok[r] = 5, -1, -1
+                break
+            a = int(np.argmax(row))
+            if i == k:
+                tok[r] = a
+                break
+            if int(batch.draft_tokens[d0 + i]) != a:
+                L[r], tok[r] = i, a
+                break
+        row0 += k + 1
+        d0 += k
+    return {"accepted_len": L, "next_token": tok, "status": st}

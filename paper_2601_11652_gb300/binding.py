@@ -56,7 +56,8 @@ _lib = None
 
 EXPORTED = ["wisp_verify_workspace_size", "wisp_verify_attention", "wisp_verify_accept", "wisp_verify_step",
             "wisp_verify_get_device_status", "wisp_verify_status_string", "wisp_verify_device_code_string",
-            "wisp_verify_accept_noalloc", "wisp_kv_workspace_size", "wisp_kv_reserve_append", "wisp_kv_commit"]
+            "wisp_verify_accept_noalloc", "wisp_verify_accept_greedy", "wisp_kv_workspace_size",
+            "wisp_kv_reserve_append", "wisp_kv_commit"]
 
 
 def lib_path() -> str:
@@ -82,6 +83,8 @@ def load(path: str | None = None):
     lib.wisp_verify_accept.restype = ctypes.c_int
     lib.wisp_verify_step.argtypes = [AP, CP, _P, ctypes.c_size_t, _P]
     lib.wisp_verify_step.restype = ctypes.c_int
+    lib.wisp_verify_accept_greedy.argtypes = [CP, _P, ctypes.c_size_t, _P]
+    lib.wisp_verify_accept_greedy.restype = ctypes.c_int
     lib.wisp_verify_accept_noalloc.argtypes = [CP, _P]
     lib.wisp_verify_accept_noalloc.restype = ctypes.c_int
     lib.wisp_verify_get_device_status.argtypes = [_P, ctypes.POINTER(_I32), ctypes.POINTER(ctypes.c_int64)]
@@ -190,6 +193,11 @@ def wisp_verify_attention(attn: wisp_attn_args, workspace: torch.Tensor, stream=
 
 def wisp_verify_accept(acc: wisp_accept_args, workspace: torch.Tensor, stream=None) -> None:
     _check("wisp_verify_accept", load().wisp_verify_accept(
+        ctypes.byref(acc), _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def wisp_verify_accept_greedy(acc: wisp_accept_args, workspace: torch.Tensor, stream=None) -> None:
+    _check("wisp_verify_accept_greedy", load().wisp_verify_accept_greedy(
         ctypes.byref(acc), _ptr(workspace), workspace.numel(), _stream(stream)))
 
 

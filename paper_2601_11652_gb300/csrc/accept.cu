@@ -734,6 +734,105 @@ __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ Acce
   cluster.sync();  // no CTA leaves while another may still read its shared memory
 }
 
+// ---- greedy (temperature 0) acceptance -----------------------------------------------------
+// Sampling at temperature 0 takes the most likely token, so the rule of Eq. 1-3 becomes: accept
+// y_i iff y_i is the argmax of logit row i-1 (the lowest token id among equal maxima), stop at the
+// first mismatch, and emit the argmax of row L.  row_argmax_kernel: one warp per (row, slice), every
+// row in parallel; greedy_walk_kernel: one warp per request merges the slices of its rows in order.
+struct RowArg {
+  float m;  // max of the slice (-inf if none)
+  int idx;  // lowest token id attaining it
+};
+
+template <typename LT>
+__global__ void __launch_bounds__(NT) row_argmax_kernel(const __grid_constant__ AcceptParams p) {
+  constexpr int E = LTraits<LT>::E;
+  const int lane = threadIdx.x & 31;
+  const int64_t unit = (int64_t)blockIdx.x * NW + (threadIdx.x >> 5);
+  if (unit >= p.total_rows * p.slices) return;
+  const int64_t row = unit / p.slices;
+  const int sl = (int)(unit % p.slices);
+  const int V = p.V;
+  const LT *rowp = static_cast<const LT *>(p.logits) + row * (int64_t)V;
+  const int64_t nvec = (V + E - 1) / E;
+  const int64_t vlo = min(nvec, (int64_t)sl * p.vps);
+  const int64_t vhi = min(nvec, vlo + p.vps);
+  float m = -INFINITY;
+  int idx = INT32_MAX;
+  // a lane visits its elements in increasing token order, so a strict ">" keeps the first maximum
+  for (int64_t vi = vlo + lane; vi < vhi; vi += 32) {
+    const uint4 w = load_vec<LT>(rowp, vi, V, p.vec_z != 0);
+#pragma unroll
+    for (int i = 0; i < E; ++i) {
+      const float z = vec_elem<LT>(w, i);
+      if (z > m) {
+        m = z;
+        idx = (int)(vi * E + i);
+      }
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    const float om = __shfl_xor_sync(0xffffffffu, m, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, idx, o);
+    if (om > m || (om == m && oi < idx)) {
+      m = om;
+      idx = oi;
+    }
+  }
+  if (lane == 0) reinterpret_cast<RowArg *>(p.parts)[unit] = RowArg{m, idx};
+}
+
+template <typename LT>
+__global__ void __launch_bounds__(NT) greedy_walk_kernel(const __grid_constant__ AcceptParams p) {
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * NW + (threadIdx.x >> 5);
+  if (r >= p.B || p.req_flag[r] != REQ_OK) return;
+  const int V = p.V, k = p.draft_lens[r], S = p.slices;
+  const int64_t Q0 = p.q_row_start[r], D0 = p.draft_start[r];
+  const RowArg *parts = reinterpret_cast<const RowArg *>(p.parts);
+  int L = k, tok = -1, err = 0;
+  for (int i = 0; i <= k; ++i) {
+    RowArg a{-INFINITY, INT32_MAX};
+    if (lane < S) a = parts[(Q0 + i) * S + lane];
+    for (int o = 16; o > 0; o >>= 1) {
+      const float om = __shfl_xor_sync(0xffffffffu, a.m, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, a.idx, o);
+      if (om > a.m || (om == a.m && oi < a.idx)) {
+        a.m = om;
+        a.idx = oi;
+      }
+    }
+    if (!(a.m > -INFINITY) || a.idx >= V) {  // no finite logit in the row
+      err = WISP_DEV_BAD_PROB;
+      break;
+    }
+    if (i == k) {
+      tok = a.idx;
+      break;
+    }
+    const int32_t y = __ldg(p.draft_tokens + D0 + i);
+    if (y < 0 || y >= V) {
+      err = WISP_DEV_BAD_TOKEN;
+      break;
+    }
+    if (y != a.idx) {
+      L = i;
+      tok = a.idx;
+      break;
+    }
+  }
+  if (lane == 0) {
+    if (err) {
+      report(p.status, err, p.request_ids, r);
+      p.accepted_len[r] = -1;
+      p.next_token[r] = -1;
+    } else {
+      p.accepted_len[r] = L;
+      p.next_token[r] = tok;
+    }
+  }
+}
+
 // ---------------------------------------------------------------------------- host side
 namespace {
 
@@ -789,6 +888,18 @@ cudaError_t accept_stats_launch(const AcceptParams &p, bool bf16, cudaStream_t s
 
 cudaError_t accept_walk_launch(const AcceptParams &p, bool bf16, cudaStream_t s) {
   return bf16 ? walk_t<uint16_t>(p, s) : walk_t<float>(p, s);
+}
+
+cudaError_t accept_greedy_launch(const AcceptParams &p, bool bf16, cudaStream_t s) {
+  const unsigned g1 = (unsigned)((p.total_rows * p.slices + NW - 1) / NW), g2 = (unsigned)((p.B + NW - 1) / NW);
+  if (bf16) {
+    row_argmax_kernel<uint16_t><<<g1, NT, 0, s>>>(p);
+    greedy_walk_kernel<uint16_t><<<g2, NT, 0, s>>>(p);
+  } else {
+    row_argmax_kernel<float><<<g1, NT, 0, s>>>(p);
+    greedy_walk_kernel<float><<<g2, NT, 0, s>>>(p);
+  }
+  return cudaGetLastError();
 }
 
 }  // namespace wisp

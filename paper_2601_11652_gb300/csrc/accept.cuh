@@ -49,5 +49,7 @@ cudaError_t accept_setup();  // once per device: shared-memory attributes
 cudaError_t accept_stats_launch(const AcceptParams &p, bool bf16, cudaStream_t s);
 // per-request walk and draw (needs the statistics and the planner's offsets)
 cudaError_t accept_walk_launch(const AcceptParams &p, bool bf16, cudaStream_t s);
+// greedy (temperature 0) variant: argmax partials of every row, then the walk (two launches)
+cudaError_t accept_greedy_launch(const AcceptParams &p, bool bf16, cudaStream_t s);
 
 }  // namespace wisp

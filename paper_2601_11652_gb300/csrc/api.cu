@@ -95,16 +95,17 @@ void accept_slices(const wisp_accept_args *c, int sms, int *slices, int *vps) {
   *slices = (int)((nvec + v - 1) / v);
 }
 
-wisp_status check_accept(const wisp_accept_args *c) {
+// need_probs: the sampling rule reads the draft distributions and the uniforms; the greedy one does not
+wisp_status check_accept(const wisp_accept_args *c, bool need_probs = true) {
   if (!c) return WISP_ERR_INVALID_ARG;
   if (c->B < 0 || c->V <= 0 || c->total_draft < 0) return WISP_ERR_INVALID_ARG;
   if (c->logits_dtype != WISP_F32 && c->logits_dtype != WISP_BF16) return WISP_ERR_INVALID_ARG;
   if (c->B == 0) return WISP_OK;
   if (c->total_q_rows < c->B) return WISP_ERR_INVALID_ARG;
-  if (!c->draft_lens || !c->target_logits || !c->sample_uniforms || !c->accepted_len || !c->next_token)
-    return WISP_ERR_INVALID_ARG;
-  if (c->total_draft > 0 && (!c->draft_tokens || !c->draft_probs || !c->accept_uniforms))
-    return WISP_ERR_INVALID_ARG;
+  if (!c->draft_lens || !c->target_logits || !c->accepted_len || !c->next_token) return WISP_ERR_INVALID_ARG;
+  if (need_probs && !c->sample_uniforms) return WISP_ERR_INVALID_ARG;
+  if (c->total_draft > 0 && !c->draft_tokens) return WISP_ERR_INVALID_ARG;
+  if (need_probs && c->total_draft > 0 && (!c->draft_probs || !c->accept_uniforms)) return WISP_ERR_INVALID_ARG;
   if (c->V > (1 << 24)) return WISP_ERR_UNSUPPORTED;  // vocabulary limit of the acceptance kernel
   if ((int64_t)c->B * 8 > INT32_MAX) return WISP_ERR_UNSUPPORTED;
   if ((int64_t)c->total_q_rows * kMaxSlices > INT32_MAX) return WISP_ERR_UNSUPPORTED;
@@ -315,7 +316,7 @@ extern "C" {
 size_t wisp_verify_workspace_size(const wisp_attn_args *attn, const wisp_accept_args *acc) {
   if (!attn && !acc) return 0;
   if (attn && check_attn(attn) != WISP_OK) return 0;
-  if (acc && check_accept(acc) != WISP_OK) return 0;
+  if (acc && check_accept(acc, false) != WISP_OK) return 0;  // the size does not depend on the distributions
   if (attn && acc && attn->B != acc->B) return 0;
   int dev = 0, sms = 0;
   if (device_setup(&dev, &sms) != WISP_OK) return 0;
@@ -346,6 +347,20 @@ wisp_status wisp_verify_accept(const wisp_accept_args *acc, void *ws, size_t ws_
   if ((st = launch_plan(nullptr, acc, ws, L, s)) != WISP_OK) return st;
   if (acc->B == 0) return WISP_OK;
   return launch_accept(acc, ws, L, sms, s);
+}
+
+wisp_status wisp_verify_accept_greedy(const wisp_accept_args *acc, void *ws, size_t ws_bytes, void *stream) {
+  wisp_status st = check_accept(acc, false);
+  if (st != WISP_OK) return st;
+  int dev = 0, sms = 0;
+  if ((st = device_setup(&dev, &sms)) != WISP_OK) return st;
+  const Layout L = make_layout(nullptr, acc, sms);
+  if ((st = check_ws(ws, ws_bytes, L)) != WISP_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((st = launch_plan(nullptr, acc, ws, L, s)) != WISP_OK) return st;
+  if (acc->B == 0) return WISP_OK;
+  const AcceptParams ap = accept_params(acc, ws, L, sms);
+  return accept_greedy_launch(ap, acc->logits_dtype == WISP_BF16, s) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
 }
 
 wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args *acc, void *ws, size_t ws_bytes,
