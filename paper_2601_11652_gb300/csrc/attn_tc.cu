@@ -61,7 +61,8 @@ struct Cfg {
   static constexpr int OFF_K = OFF_Q + 2 * Q_BYTES;
   static constexpr int OFF_V = OFF_K + NSTAGE * KV_TILE;
   static constexpr int OFF_P = OFF_V + NSTAGE * KV_TILE;
-  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+  static constexpr int NPBUF = 3;                // P buffers: P(n) in buffer n % 3
+  static constexpr int OFF_BAR = OFF_P + NPBUF * P_BYTES;
   static constexpr int N_BAR = 4 * NSTAGE + 24 + 2 * RING;
   static constexpr int OFF_RED = OFF_BAR + N_BAR * 8;        // float [2][128] row sums (epilogue)
   static constexpr int OFF_MISC = OFF_RED + 2 * 128 * 4;     // tmem base, flags
@@ -122,9 +123,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   B.q_empty = B.q_full + 2;
   B.s_full = B.q_empty + 2;
   B.s_empty = B.s_full + 2;
-  B.p_full = B.s_empty + 2;
-  B.o_full = B.p_full + 2;  // [2]: PV of even / odd tiles
-  B.o_empty = B.o_full + 2;  // [2] per O buffer: its epilogue is done
+  B.p_full = B.s_empty + 2;  // [3] per P buffer
+  B.o_full = B.p_full + 3;  // [3] per P buffer: PV of tiles n with n % 3 == b
+  B.o_empty = B.o_full + 3;  // [2] per O buffer: its epilogue is done
   B.o_done = B.o_empty + 2;  // [2] per O buffer: the item's last PV is done
   B.ep_full = B.o_done + 2;  // [2] per O buffer: the softmax warps handed the item over
   B.mma_done = B.ep_full + 2;
@@ -156,10 +157,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::mbar_init(B.q_empty + b, 1);
       ptx::mbar_init(B.s_full + b, 1);
       ptx::mbar_init(B.s_empty + b, 4);
+    }
+    for (int b = 0; b < 3; ++b) {
       ptx::mbar_init(B.p_full + b, 4);
+      ptx::mbar_init(B.o_full + b, 1);
     }
     for (int b = 0; b < 2; ++b) {
-      ptx::mbar_init(B.o_full + b, 1);
       ptx::mbar_init(B.o_empty + b, 4);  // the four epilogue warps
       ptx::mbar_init(B.o_done + b, 1);
       ptx::mbar_init(B.ep_full + b, 4);  // the four softmax warps
@@ -388,11 +391,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         if (n_pv < n_s) {
-          const int pb = n_pv & 1;
+          const int pb = (int)(n_pv % 3);
           const bool first = tflag[n_pv & 3] & 1, last = tflag[n_pv & 3] & 2;
           const int tl = tli[n_pv & 3], ob = tl & 1;  // the item's O buffer
           const int st = (int)(n_pv % C::NSTAGE);
-          if (ptx::mbar_test_wait(B.p_full + pb, (n_pv >> 1) & 1) &&
+          if (ptx::mbar_test_wait(B.p_full + pb, (n_pv / 3) & 1) &&
               ptx::mbar_test_wait(B.v_full + st, (n_pv / C::NSTAGE) & 1) &&
               (!first || ptx::mbar_test_wait(B.o_empty + ob, ((tl >> 1) & 1) ^ 1))) {
             ptx::tc_fence_after();
@@ -404,7 +407,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const uint64_t b = ptx::sdesc_sw128(va + ks * 16 * 128, kBN * 128, 1024);
               ptx::umma_f16(tmem + 128 + ob * 128, a, b, IDESC_PV, (!first || ks > 0) ? 1u : 0u);
             }
-            ptx::umma_commit(B.o_full + (n_pv & 1));
+            ptx::umma_commit(B.o_full + pb);
             ptx::umma_commit(B.v_empty + st);
             if (last) ptx::umma_commit(B.o_done + ob);
             ++n_pv;
@@ -650,19 +653,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int i = 0; i < CW; ++i) sv[i] = sr[i] * scale_log2;  // -inf stays -inf
           } else {
-            // this warp's own CW columns, read again from TMEM (cheaper than selecting registers)
-            uint32_t x[CW];
-            if constexpr (CW == 16) {
-              ptx::tmem_ld16(tmem + lane_addr + sb * 64 + c0, x);
-            } else {
-              ptx::tmem_ld32(tmem + lane_addr + sb * 64 + c0, x);
-            }
-            ptx::tmem_wait_ld();
+            // this warp's own CW columns, taken from the (already masked) row in registers; the
+            // replica index is warp-uniform, so each case reads registers at constant indices
+            auto take = [&](auto part) {
+              constexpr int o = decltype(part)::value * CW;
 #pragma unroll
-            for (int i = 0; i < CW; ++i) {
-              const int tok = tok0 + c0 + i;
-              const bool ok_tok = interior || (tok < w.t1 && tok <= vis);
-              sv[i] = ok_tok ? __uint_as_float(x[i]) * scale_log2 : -INFINITY;
+              for (int i = 0; i < CW; ++i) sv[i] = sr[o + i] * scale_log2;
+            };
+            const int part = c0 / CW;
+            if (part == 0) take(std::integral_constant<int, 0>{});
+            else if (part == 1) take(std::integral_constant<int, 1>{});
+            if constexpr (CW == 16) {
+              if (part == 2) take(std::integral_constant<int, 2>{});
+              else if (part == 3) take(std::integral_constant<int, 3>{});
             }
           }
           // S(n) has been read: its TMEM buffer may be overwritten by S(n+2)
@@ -692,14 +695,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < CW; i += 2 * w2) ev[i] += ev[i + w2];
           }
           l += ev[0];
-          // PV(m) completes barrier o_full[m & 1] for the (m >> 1)-th time.  Every softmax warp
-          // waits PV(n-2) here (P buffer n & 1 is free again); since it waited PV(n-4) two tiles
-          // ago and PV(n) needs the P(n) it is about to publish, the parity names exactly PV(n-2).
-          if (n >= 2 && !wait_bar(B.o_full + (n & 1), ((n - 2) >> 1) & 1, s_abort)) return false;
+          // PV(m) completes barrier o_full[m % 3] for the (m / 3)-th time.  Every softmax warp
+          // waits PV(n-3) here (P buffer n % 3 is free again); since it waited PV(n-6) three tiles
+          // ago and PV(n) needs the P(n) it is about to publish, the parity names exactly PV(n-3).
+          const int pbuf = (int)(n % 3);
+          if (n >= 3 && !wait_bar(B.o_full + pbuf, ((n - 3) / 3) & 1, s_abort)) return false;
           // a rescale of the O rows needs PV(n-1) complete (exact for the same reason) and
           // precedes PV(n); each warp rescales its own column slice of its quadrant's rows
           if (t > 0 && __ballot_sync(0xffffffffu, rescale)) {
-            if (!wait_bar(B.o_full + ((n - 1) & 1), ((n - 1) >> 1) & 1, s_abort)) return false;
+            if (!wait_bar(B.o_full + (n - 1) % 3, ((n - 1) / 3) & 1, s_abort)) return false;
             ptx::tc_fence_after();
             for (int c = 0; c < dcw; c += 16) {
               uint32_t x[16];
@@ -715,7 +719,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // this warp's columns of P row `row` (bf16, 128-byte swizzle)
 #pragma unroll
           for (int rr = 0; rr < kBN / CW; ++rr) {
-            uint8_t *prow = smem + C::OFF_P + sb * C::P_BYTES + (rr * G + row) * 128;  // (rr*G + row) & 7 == row & 7
+            uint8_t *prow = smem + C::OFF_P + pbuf * C::P_BYTES + (rr * G + row) * 128;  // (rr*G + row) & 7 == row & 7
 #pragma unroll
             for (int c = 0; c < CW / 8; ++c) {
               const int cc = c0 / 8 + c;
@@ -725,7 +729,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           ptx::fence_proxy_async_smem();
           __syncwarp();
-          if (lane == 0) ptx::mbar_arrive(B.p_full + sb);
+          if (lane == 0) ptx::mbar_arrive(B.p_full + pbuf);
         }
         return true;
       };
