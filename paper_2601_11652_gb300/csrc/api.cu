@@ -128,11 +128,14 @@ Layout make_layout(const wisp_attn_args *a, const wisp_accept_args *c, int sms) 
   L.plan_header = take(sizeof(PlanHeader));
   if (a) {
     L.target_items = sms * kItemsPerSM;
-    L.max_items = (int64_t)L.target_items + (int64_t)B * a->Hkv;
+    // the tensor-core kernel takes at most kTcRowsPerItem query rows per item: a (request, head)
+    // with more is cut into two row groups, which at most doubles the item count
+    const int64_t rg = a->qkv_dtype == WISP_BF16 ? 2 : 1;
+    L.max_items = rg * ((int64_t)L.target_items + (int64_t)B * a->Hkv);
     L.partial_cap = (int64_t)2 * L.target_items * kMaxRowsPerHead * (a->D + 2);
     L.req_item_begin = take(sizeof(int32_t) * (size_t)B);
     L.req_chunks = take(sizeof(int32_t) * (size_t)B);
-    L.pair_done = take(sizeof(int32_t) * (size_t)B * a->Hkv);
+    L.pair_done = take(sizeof(int32_t) * (size_t)B * a->Hkv * 2);
     L.items = take(sizeof(WorkItem) * (size_t)L.max_items);
     L.order = take(sizeof(int32_t) * (size_t)L.max_items);
     L.partials = take(sizeof(float) * (size_t)L.partial_cap);
@@ -178,6 +181,7 @@ PlanParams plan_params(const wisp_attn_args *a, const wisp_accept_args *c, void 
     pp.context_lens = a->context_lens;
     pp.with_attention = 1;
     pp.target_items = L.target_items;
+    pp.max_rows_item = a->qkv_dtype == WISP_BF16 ? kTcRowsPerItem : kMaxRowsPerHead;
     pp.max_items = L.max_items;
     pp.partial_cap = L.partial_cap;
     pp.req_item_begin = at<int32_t>(ws, L.req_item_begin);

@@ -3,34 +3,39 @@
 // Same contract as attn_simt.cu (Sec. 4.4-4.5: request r's k+1 new queries over its
 // L_total = L_cached + L_new paged keys, query j seeing keys 0..c_r + j), built for sm_103a.
 //
-// Persistent CTAs (one per SM) take work items (request, KV head, key chunk) from a global
-// counter, in the planner's longest-first order.  Warp roles in a CTA:
-//   * warp 6 (item loader) takes the next item, publishes it to the other warps through a
-//     4-slot shared ring, and copies its query rows into one of two shared Q buffers
-//     (128-byte-swizzled K-major layout);
-//   * warps 0 and 7 (K and V producers) stream the item's K and V tiles of 64 tokens with TMA
-//     tiled loads into two separate rings, one 8 KB box per 64-wide half of the head dim when
-//     the tile's four 16-token blocks are consecutive in the pool, else one 2 KB box per block;
-//     blocks past the item read as zeros (out-of-range box).  A K stage is free again once S of
-//     its tile is done, a V stage once PV is;
-//   * warp 1 (one thread) issues tcgen05.mma: S = Q K^T (M = 128, N = 64, K = D) into one of two
-//     TMEM tiles, and O += P V (M = 128, N = D, K = 64) into the item's TMEM accumulator (two
-//     accumulators, alternating between items);
-//   * warps 2-5 (softmax): the g*(k+1) query rows of an item are placed in a row group of
-//     G = 32, 64 or 128 MMA rows and replicated 128/G times, so that each of the four TMEM lane
-//     quadrants holds a copy.  Each warp reads the whole 64-column S row of its lane (so the
-//     replicas agree on the row max without talking to each other) and handles 64/rep of the
-//     columns: exponentials, its share of the row sum, and P (bf16, swizzled, written to every
-//     replica row) for the PV product.  The reference max only moves when a tile max exceeds it
-//     by more than 2^8 (then the warp rescales its slice of the O rows in TMEM), so
-//     P = 2^(s - m_ref) <= 2^8.  At the item's end the row-sum share and the max go to spare
-//     TMEM columns and the item is handed over;
-//   * warps 8-11 (epilogue) add the row-sum shares, read O from TMEM and write the normalised
+// A verification item has few query rows (g * (k+1), at most 64 per item) and many keys, so the
+// products run transposed: the keys are the MMA's M dimension and the query rows its N.
+//   S^T = K Q^T       (M = 128 keys of a tile, N = the item's rows rounded up to 16, K = D)
+//   O^T += V^T P^T    (M = D, N = rows, K = 128 keys)
+// Nothing is replicated to fill the 128-row MMA, and the tensor core reads each K and V tile from
+// shared memory once.
+//
+// Persistent CTAs (one per SM) take work items (request, KV head, key chunk, row group) from a
+// global counter, in the planner's longest-first order.  Warp roles in a CTA:
+//   * warp 6 (item loader) takes the next item, publishes it to the other warps through a 4-slot
+//     shared ring, and copies its query rows into one of two shared Q buffers (128-byte-swizzled,
+//     K-major: the B operand of S^T);
+//   * warps 0 and 7 (K and V producers) stream the item's K and V tiles of 128 tokens with TMA
+//     tiled loads into two rings: one 16 KB box per 64-wide half of the head dim when the tile's
+//     eight 16-token blocks are consecutive in the pool, else one 2 KB box per block; blocks past
+//     the item read as zeros (out-of-range box).  A K stage is free again once S^T of its tile is
+//     done, a V stage once its PV product is;
+//   * warp 1 (one thread) issues tcgen05.mma: S^T into one of two TMEM tiles (key t in TMEM lane
+//     t, query row j in column j), and O^T into the item's TMEM accumulator (head-dim index d in
+//     lane d, row j in column j; two accumulators alternating between items);
+//   * warps 2-5 (softmax), one per TMEM lane quadrant, i.e. 32 keys of each tile per warp: a thread
+//     holds one key's scores for all rows.  The rows' reference maxima live in shared memory; a
+//     tile whose scores exceed a reference by more than 2^8 anywhere (the first tile of an item
+//     always does) makes the four warps agree on new maxima (exact per-row tile maxima) and, if O
+//     holds earlier tiles, rescale the O^T columns in TMEM.  Each thread writes its key's P row
+//     (bf16, MN-major, swizzled: the B operand of the PV product) and keeps its share of every
+//     row sum;
+//   * warps 8-11 (epilogue) add the row-sum shares, read O^T from TMEM and write the normalised
 //     output or, for a split item, the (O, m, l) partials; the last chunk of a split
-//     (request, head) to finish merges all its chunks.  This runs while the softmax warps are
-//     already on the next item.
-// Every mbarrier wait is bounded in time; an expired wait records WISP_DEV_TIMEOUT and the
-// CTA drains.  Rows past g*(k+1) are padding: computed from stale data, never written.
+//     (request, head, row group) to finish merges all its chunks.  This runs while the softmax
+//     warps are already on the next item.
+// Every mbarrier wait is bounded in time; an expired wait records WISP_DEV_TIMEOUT and the CTA
+// drains.  No named barrier is used: a warp that gives up cannot leave the others blocked.
 #include "attn.cuh"
 #include "sm100_ptx.cuh"
 
@@ -41,41 +46,52 @@ namespace wisp {
 
 namespace {
 
-constexpr int kBN = 64;             // KV tokens per tile
-constexpr int kM = 128;             // MMA rows
+constexpr int kBT = 128;            // KV tokens per tile (the M of S^T)
+constexpr int kNR = kTcRowsPerItem; // query rows per item at most (64: the planner cuts larger sets)
 constexpr int kThreads = 384;       // warp 0 K producer, warp 1 MMA, warps 2-5 softmax, warp 6 item loader,
                                     // warp 7 V producer, warps 8-11 epilogue
-constexpr uint32_t kTmemCols = 512; // S[2] at columns 0 / 64, O[2] at 128 / 256, (l, m) hand-over at 384
+constexpr uint32_t kTmemCols = 256; // S^T[2] at columns 0 / 64, O^T[2] at 128 / 192
 constexpr long long kWaitCycles = 4000000000LL;  // about two seconds: a wait that long is a failure
 constexpr float kTau = 8.0f;        // lazy rescale threshold (log2 units)
+constexpr float kExpTau = 256.0f;   // 2^kTau
+static_assert(kNR == 64, "TMEM and shared-memory layout assume 64 rows per item");
 
 template <int D>
 struct Cfg {
   static constexpr int HALVES = D / 64;
-  static constexpr int Q_BYTES = kM * D * 2;
-  static constexpr int KV_TILE = kBN * D * 2;  // K (or V) of one tile
-  static constexpr int NSTAGE = D == 128 ? 3 : 6;
-  static constexpr int P_BYTES = kM * kBN * 2;
-  static constexpr int RING = 4;               // slots of the item ring
+  static constexpr int HALF = kBT * 128;        // one 64-wide half of a K / V tile: [128 tokens][128 B]
+  static constexpr int KV_TILE = HALVES * HALF; // K (or V) of one tile
+  static constexpr int QHALF = kNR * 128;       // one half of a Q buffer: [64 rows][128 B]
+  static constexpr int Q_BYTES = HALVES * QHALF;
+  static constexpr int P_BYTES = kBT * kNR * 2; // P^T: [128 tokens][64 rows] bf16
+  static constexpr int NSK = D == 128 ? 2 : 4;  // K ring stages
+  static constexpr int NSV = D == 128 ? 2 : 4;  // V ring stages
+  static constexpr int NP = 2;                  // P buffers: P(n) in buffer n % NP
+  static constexpr int RING = 4;                // slots of the item ring
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = OFF_Q + 2 * Q_BYTES;
-  static constexpr int OFF_V = OFF_K + NSTAGE * KV_TILE;
-  static constexpr int OFF_P = OFF_V + NSTAGE * KV_TILE;
-  static constexpr int NPBUF = 3;                // P buffers: P(n) in buffer n % 3
-  static constexpr int OFF_BAR = OFF_P + NPBUF * P_BYTES;
-  static constexpr int N_BAR = 4 * NSTAGE + 24 + 2 * RING;
-  static constexpr int OFF_RED = OFF_BAR + N_BAR * 8;        // float [2][128] row sums (epilogue)
-  static constexpr int OFF_MISC = OFF_RED + 2 * 128 * 4;     // tmem base, flags
-  static constexpr int OFF_RING = OFF_MISC + 64;             // RING x (index, WorkItem)
-  static constexpr int SMEM = OFF_RING + RING * 48 + 1024;   // + slack to align the base to 1024
+  static constexpr int OFF_V = OFF_K + NSK * KV_TILE;
+  static constexpr int OFF_P = OFF_V + NSV * KV_TILE;
+  static constexpr int OFF_BAR = OFF_P + NP * P_BYTES;
+  static constexpr int N_BAR = 2 * NSK + 2 * NSV + 8 + 2 * NP + 6 + 1 + 2 * RING + 5;
+  static constexpr int OFF_MW = (OFF_BAR + N_BAR * 8 + 15) / 16 * 16;  // float [4][64] per-warp row maxima
+  static constexpr int OFF_FW = OFF_MW + 4 * kNR * 4;                  // float [4][64] per-warp rescale factors
+  static constexpr int OFF_RED = OFF_FW + 4 * kNR * 4;                 // float [4][64] tile maxima per warp
+  static constexpr int OFF_FLAG = OFF_RED + 4 * kNR * 4;               // uint32 [2][4] exceed flags per warp
+  static constexpr int OFF_HL = OFF_FLAG + 32;                         // float [2][4][64] row-sum shares per warp
+  static constexpr int OFF_HM = OFF_HL + 2 * 4 * kNR * 4;              // float [2][64] row reference maxima
+  static constexpr int OFF_EM = OFF_HM + 2 * kNR * 4;                  // float [2][64] merge: max, 1 / sum
+  static constexpr int OFF_TR = OFF_EM + 2 * kNR * 4;                  // float [4][32][33] per-warp transposes
+  static constexpr int OFF_MISC = OFF_TR + 4 * 32 * 33 * 4;            // tmem base, flags
+  static constexpr int OFF_RING = OFF_MISC + 64;                       // RING x (index, WorkItem)
+  static constexpr int SMEM = OFF_RING + RING * 64 + 1024;             // + slack to align the base to 1024
   static_assert(SMEM <= 227 * 1024, "shared memory of one CTA on sm_103a");
+  static_assert(OFF_K % 1024 == 0 && OFF_V % 1024 == 0 && OFF_P % 1024 == 0, "swizzled buffers need 1 KB alignment");
 };
-
-constexpr uint32_t IDESC_S = ptx::idesc_bf16_f32(kM, kBN, false);
 
 struct Bars {
   uint64_t *k_full, *k_empty, *v_full, *v_empty, *q_full, *q_empty, *s_full, *s_empty, *p_full, *o_full;
-  uint64_t *o_empty, *o_done, *ep_full, *mma_done, *it_full, *it_empty, *egrp;
+  uint64_t *o_empty, *o_done, *ep_full, *mma_done, *it_full, *it_empty, *egrp, *sm_sync, *sm_sync2, *fin, *claim;
 };
 
 __device__ __forceinline__ bool wait_bar(uint64_t *b, uint32_t parity, volatile int *abort) {
@@ -92,14 +108,27 @@ __device__ __forceinline__ bool wait_bar(uint64_t *b, uint32_t parity, volatile 
 }
 
 __device__ __forceinline__ bool item_ok(const AttnParams &p, const WorkItem &w) {
-  return w.r >= 0 && w.r < p.B && p.req_flag[w.r] == REQ_OK && w.t1 > w.t0 && w.rows > 0 && w.rows <= kM;
+  return w.r >= 0 && w.r < p.B && p.req_flag[w.r] == REQ_OK && w.t1 > w.t0 && w.rows > 0 && w.rows <= kNR &&
+         w.row0 >= 0 && (w.nrg == 1 || w.nrg == 2) && w.rg >= 0 && w.rg < w.nrg;
 }
-
-__device__ __forceinline__ int row_group(int rows) { return rows <= 32 ? 32 : (rows <= 64 ? 64 : 128); }
 
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// Reductions over the 32 lanes of a warp through a padded shared 32 x 33 scratch: on return lane i
+// holds the sum (max) over all lanes of v[i].  Conflict-free both ways.
+template <bool MAX>
+__device__ __forceinline__ float warp_transpose_reduce(const float (&v)[32], float *tr, int lane) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i) tr[lane * 33 + i] = v[i];
+  __syncwarp();
+  float r = MAX ? -INFINITY : 0.0f;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) r = MAX ? fmaxf(r, tr[i * 33 + lane]) : r + tr[i * 33 + lane];
+  __syncwarp();
+  return r;
 }
 
 }  // namespace
@@ -107,8 +136,8 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ AttnParams p, const __grid_constant__ CUtensorMap tmk,
-                   const __grid_constant__ CUtensorMap tmv, const __grid_constant__ CUtensorMap tmk4,
-                   const __grid_constant__ CUtensorMap tmv4) {
+                   const __grid_constant__ CUtensorMap tmv, const __grid_constant__ CUtensorMap tmk8,
+                   const __grid_constant__ CUtensorMap tmv8) {
   using C = Cfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -116,23 +145,35 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t *bar = reinterpret_cast<uint64_t *>(smem + C::OFF_BAR);
   Bars B;
   B.k_full = bar;
-  B.k_empty = bar + C::NSTAGE;
-  B.v_full = bar + 2 * C::NSTAGE;
-  B.v_empty = bar + 3 * C::NSTAGE;
-  B.q_full = bar + 4 * C::NSTAGE;
+  B.k_empty = B.k_full + C::NSK;
+  B.v_full = B.k_empty + C::NSK;
+  B.v_empty = B.v_full + C::NSV;
+  B.q_full = B.v_empty + C::NSV;
   B.q_empty = B.q_full + 2;
   B.s_full = B.q_empty + 2;
   B.s_empty = B.s_full + 2;
-  B.p_full = B.s_empty + 2;  // [3] per P buffer
-  B.o_full = B.p_full + 3;  // [3] per P buffer: PV of tiles n with n % 3 == b
-  B.o_empty = B.o_full + 3;  // [2] per O buffer: its epilogue is done
-  B.o_done = B.o_empty + 2;  // [2] per O buffer: the item's last PV is done
-  B.ep_full = B.o_done + 2;  // [2] per O buffer: the softmax warps handed the item over
+  B.p_full = B.s_empty + 2;     // [NP] per P buffer
+  B.o_full = B.p_full + C::NP;  // [NP] per P buffer: PV of tiles n with n % NP == b
+  B.o_empty = B.o_full + C::NP; // [2] per O buffer: its epilogue is done
+  B.o_done = B.o_empty + 2;     // [2] per O buffer: the item's last PV is done
+  B.ep_full = B.o_done + 2;     // [2] per O buffer: the softmax warps handed the item over
   B.mma_done = B.ep_full + 2;
   B.it_full = B.mma_done + 1;
   B.it_empty = B.it_full + C::RING;
   B.egrp = B.it_empty + C::RING;
-  float *s_lsum = reinterpret_cast<float *>(smem + C::OFF_RED);  // [2][128]
+  B.sm_sync = B.egrp + 1;       // the four softmax warps, once per tile
+  B.sm_sync2 = B.sm_sync + 1;   // the four softmax warps, once per tile that moves a reference max
+  B.fin = B.sm_sync2 + 1;       // every warp, once: its last access to TMEM is done
+  B.claim = B.fin + 1;          // the K producer, once per item, a few tiles before the item's end
+  static_assert(2 * C::NSK + 2 * C::NSV + 8 + 2 * C::NP + 6 + 1 + 2 * C::RING + 5 <= C::N_BAR, "barrier count");
+  float *s_mw = reinterpret_cast<float *>(smem + C::OFF_MW);
+  float *s_fw = reinterpret_cast<float *>(smem + C::OFF_FW);
+  float *s_red = reinterpret_cast<float *>(smem + C::OFF_RED);
+  volatile uint32_t *s_flag = reinterpret_cast<volatile uint32_t *>(smem + C::OFF_FLAG);
+  float *s_em = reinterpret_cast<float *>(smem + C::OFF_EM);
+  float *s_hl = reinterpret_cast<float *>(smem + C::OFF_HL);
+  float *s_hm = reinterpret_cast<float *>(smem + C::OFF_HM);
+  float *s_tr = reinterpret_cast<float *>(smem + C::OFF_TR);
   uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + C::OFF_MISC);
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + C::OFF_MISC + 4);
   volatile int *s_last = reinterpret_cast<volatile int *>(smem + C::OFF_MISC + 8);
@@ -141,14 +182,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     int pad[3];
     WorkItem w;
   };
+  static_assert(sizeof(RingSlot) <= 64, "item ring slot");
   RingSlot *s_ring = reinterpret_cast<RingSlot *>(smem + C::OFF_RING);
-  static_assert(C::OFF_RING + C::RING * sizeof(RingSlot) + 1024 <= C::SMEM, "item ring overflows its region");
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < C::NSTAGE; ++s) {
+    for (int s = 0; s < C::NSK; ++s) {
       ptx::mbar_init(B.k_full + s, 1);
       ptx::mbar_init(B.k_empty + s, 1);
+    }
+    for (int s = 0; s < C::NSV; ++s) {
       ptx::mbar_init(B.v_full + s, 1);
       ptx::mbar_init(B.v_empty + s, 1);
     }
@@ -158,7 +201,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::mbar_init(B.s_full + b, 1);
       ptx::mbar_init(B.s_empty + b, 4);
     }
-    for (int b = 0; b < 3; ++b) {
+    for (int b = 0; b < C::NP; ++b) {
       ptx::mbar_init(B.p_full + b, 4);
       ptx::mbar_init(B.o_full + b, 1);
     }
@@ -172,15 +215,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::mbar_init(B.it_full + i, 1);
       ptx::mbar_init(B.it_empty + i, 11);  // KV producers, MMA thread, softmax and epilogue warps
     }
-    ptx::mbar_init(B.egrp, 4);  // the four epilogue warps
+    ptx::mbar_init(B.egrp, 4);      // the four epilogue warps
+    ptx::mbar_init(B.sm_sync, 4);   // the four softmax warps
+    ptx::mbar_init(B.sm_sync2, 4);
+    ptx::mbar_init(B.fin, kThreads / 32);
+    ptx::mbar_init(B.claim, 1);
     *s_abort = 0;
     ptx::fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
     ptx::prefetch_tmap(&tmk);
     ptx::prefetch_tmap(&tmv);
-    ptx::prefetch_tmap(&tmk4);
-    ptx::prefetch_tmap(&tmv4);
+    ptx::prefetch_tmap(&tmk8);
+    ptx::prefetch_tmap(&tmv8);
   }
   __syncwarp();
   if (warp == 1) {
@@ -197,11 +244,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0 || warp == 7) {
     // ------------------------------------------------------------------ K / V producers
-    // K and V have rings of their own: a K stage is free again once S of its tile is done, a V
-    // stage once PV is, so each tensor is fetched about NSTAGE tiles ahead of its use.
+    // K and V have rings of their own: a K stage is free again once S^T of its tile is done, a V
+    // stage once PV is, so each tensor is fetched about as many tiles ahead of its use as its ring
+    // has stages.
     const bool is_k = warp == 0;
+    const uint32_t ns = is_k ? C::NSK : C::NSV;
     const CUtensorMap *tm1 = is_k ? &tmk : &tmv;
-    const CUtensorMap *tm4 = is_k ? &tmk4 : &tmv4;
+    const CUtensorMap *tm8 = is_k ? &tmk8 : &tmv8;
     const uint32_t off_t = sbase + (is_k ? C::OFF_K : C::OFF_V);
     uint64_t *full = is_k ? B.k_full : B.v_full;
     uint64_t *empty = is_k ? B.k_empty : B.v_empty;
@@ -221,37 +270,42 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int i = base + lane;
         return i < nblk ? __ldg(bt + i) : -1;
       };
-      int cur = fetch(0), nxt = fetch(32);
-      const int ntiles = (w.t1 - w.t0 + kBN - 1) / kBN;
+      int cur = fetch(0), nxt = fetch(32);  // block ids of tiles t..t+3 and t+4..t+7
+      const int ntiles = (w.t1 - w.t0 + kBT - 1) / kBT;
+      const int t_claim = ntiles > 3 ? ntiles - 3 : 0;
       for (int t = 0; t < ntiles; ++t, ++tile_n) {
-        if (t > 0 && (t & 7) == 0) {
+        // a few tiles before this item's end the loader may take the next one (items are taken
+        // just in time, so the work counter balances the CTAs to the end)
+        if (is_k && t == t_claim && lane == 0) ptx::mbar_arrive(B.claim);
+        if (t > 0 && (t & 3) == 0) {
           cur = nxt;
-          nxt = fetch(32 * ((t >> 3) + 1));
+          nxt = fetch(32 * ((t >> 2) + 1));
         }
-        const int s = (int)(tile_n % C::NSTAGE);
-        const uint32_t round = tile_n / C::NSTAGE;
+        const int s = (int)(tile_n % ns);
+        const uint32_t round = tile_n / ns;
         if (!wait_bar(empty + s, (round & 1) ^ 1, s_abort)) { ok = false; break; }
         if (lane == 0) ptx::mbar_arrive_expect_tx(full + s, C::KV_TILE);
         __syncwarp();
-        int bid = __shfl_sync(0xffffffffu, cur, (4 * t + (lane & 3)) & 31);
-        const int rel = 4 * t + (lane & 3);
+        const int bi = lane & 7;  // block of the tile this lane looks after
+        int bid = __shfl_sync(0xffffffffu, cur, (8 * t + bi) & 31);
+        const int rel = 8 * t + bi;
         bool valid = rel < nblk && bid >= 0 && bid < p.num_blocks;
-        if (is_k && lane < 4 && rel < nblk && !valid) report(p.status, WISP_DEV_BAD_BLOCK, p.request_ids, w.r);
+        if (is_k && lane < 8 && rel < nblk && !valid) report(p.status, WISP_DEV_BAD_BLOCK, p.request_ids, w.r);
         const int b0 = __shfl_sync(0xffffffffu, bid, 0);
-        // four consecutive valid blocks: one 8 KB box per (tensor, half) with the 4-block maps
-        const unsigned contig = __ballot_sync(0xffffffffu, lane < 4 && valid && bid == b0 + lane);
-        if (contig == 0xFu) {
+        // eight consecutive valid blocks: one 16 KB box per (tensor, half) with the 8-block maps
+        const unsigned contig = __ballot_sync(0xffffffffu, lane < 8 && valid && bid == b0 + lane);
+        if (contig == 0xFFu) {
           if (lane == 0) {
 #pragma unroll
             for (int hf = 0; hf < C::HALVES; ++hf) {
-              ptx::tma_load_4d(off_t + s * C::KV_TILE + hf * (kBN * 128), tm4, full + s, hf * 64, 0, w.h, b0);
+              ptx::tma_load_4d(off_t + s * C::KV_TILE + hf * C::HALF, tm8, full + s, hf * 64, 0, w.h, b0);
             }
           }
-        } else if (lane < 4) {
+        } else if (lane < 8) {
           if (!valid) bid = p.num_blocks;  // past the item (or invalid): out-of-range box, reads zeros
 #pragma unroll
           for (int hf = 0; hf < C::HALVES; ++hf) {
-            const uint32_t off = s * C::KV_TILE + hf * (kBN * 128) + lane * (16 * 128);
+            const uint32_t off = s * C::KV_TILE + hf * C::HALF + lane * (16 * 128);
             ptx::tma_load_4d(off_t + off, tm1, full + s, hf * 64, 0, w.h, bid);
           }
         }
@@ -260,10 +314,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!ok && lane == 0) report(p.status, WISP_DEV_TIMEOUT, p.request_ids, 0);
     // drain: every stage issued must land before the CTA's shared memory goes away
     if (lane == 0) {
-      for (uint32_t k = 0; k < (uint32_t)C::NSTAGE && k < tile_n; ++k) {
+      for (uint32_t k = 0; k < ns && k < tile_n; ++k) {
         const uint32_t n = tile_n - 1 - k;
         const long long t0 = clock64();
-        while (!ptx::mbar_try_wait(full + n % C::NSTAGE, (n / C::NSTAGE) & 1) && clock64() - t0 < kWaitCycles) {
+        while (!ptx::mbar_try_wait(full + n % ns, (n / ns) & 1) && clock64() - t0 < kWaitCycles) {
         }
       }
     }
@@ -272,8 +326,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     int li = 0;
     bool ok = true;
     for (uint32_t j = 0; ok; ++j) {
-      // next valid work item: publish it to the other warps, then load its query rows
+      // next valid work item: publish it to the other warps, then load its query rows.  Item j is
+      // taken once the K producer is near the end of item j - 1 (the claim barrier completes once
+      // per item, and the producer cannot pass item j - 1 before item j is published: the parity
+      // is exact).
       const int slot = j % C::RING;
+      if (j > 0 && !wait_bar(B.claim, (j - 1) & 1, s_abort)) { ok = false; break; }
       if (!wait_bar(B.it_empty + slot, ((j / C::RING) & 1) ^ 1, s_abort)) { ok = false; break; }
       int it = -1;
       if (lane == 0) {
@@ -293,13 +351,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int qb = li & 1;
       if (!wait_bar(B.q_empty + qb, ((li >> 1) & 1) ^ 1, s_abort)) { ok = false; break; }
       ++li;
-      // query rows of this KV head -> Q[qb]: row rho = j*g + hh, copied to MMA rows rr*G + rho.
-      // Loads are issued QBATCH at a time per lane before any store.
-      const int G = row_group(w.rows), rep = kM / G;
+      // the item's query rows -> Q[qb], row rho (query row row0 + rho = j*g + hh) at MMA row rho.
+      // Loads are issued QBATCH at a time per lane before any store.  Rows past `rows` up to the
+      // MMA's N only feed S^T columns that the softmax masks.
       const uint16_t *qg = static_cast<const uint16_t *>(p.q);
       uint8_t *qs = smem + C::OFF_Q + qb * C::Q_BYTES;
       constexpr int CPR = D / 8;  // 16-byte chunks per row
-      constexpr int QBATCH = 16;
+      constexpr int QBATCH = 8;
       const int nchunks = w.rows * CPR;
       for (int base = 0; base < nchunks; base += 32 * QBATCH) {
         uint4 v[QBATCH];
@@ -308,7 +366,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int c = base + u * 32 + lane;
           if (c < nchunks) {
             const int row = c / CPR, cc = c % CPR;
-            const int jj = row / g, hh = row % g;
+            const int rj = w.row0 + row;
+            const int jj = rj / g, hh = rj % g;
             v[u] = __ldg(reinterpret_cast<const uint4 *>(qg + ((int64_t)(w.q0 + jj) * p.Hq + w.h * g + hh) * D) + cc);
           }
         }
@@ -317,10 +376,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int c = base + u * 32 + lane;
           if (c < nchunks) {
             const int row = c / CPR, cc = c % CPR;
-            for (int rr = 0; rr < rep; ++rr) {
-              const int m = rr * G + row;
-              *reinterpret_cast<uint4 *>(qs + (cc >> 3) * (kM * 128) + m * 128 + (((cc & 7) ^ (m & 7)) << 4)) = v[u];
-            }
+            *reinterpret_cast<uint4 *>(qs + (cc >> 3) * C::QHALF + row * 128 + (((cc & 7) ^ (row & 7)) << 4)) = v[u];
           }
         }
       }
@@ -331,17 +387,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!ok && lane == 0) report(p.status, WISP_DEV_TIMEOUT, p.request_ids, 0);
   } else if (warp == 1) {
     // ------------------------------------------------------------------ MMA issuer
-    // One thread polls two queues: S(n) is issued as soon as tile n has landed, its Q is loaded
-    // and its TMEM buffer has been read; PV(m) as soon as P(m) is published (and, for an item's
-    // first tile, the previous item's O has been read).  S therefore runs ahead of PV instead of
-    // waiting behind it.
+    // One thread polls two queues: S^T(n) is issued as soon as tile n's K has landed, its Q is
+    // loaded and its TMEM buffer has been read; PV(m) as soon as P(m) is published and V(m) has
+    // landed (and, for an item's first tile, the previous item's O has been read).  S^T therefore
+    // runs ahead of PV instead of waiting behind it.
     if (lane == 0) {
-      constexpr uint32_t IDESC_PV = ptx::idesc_bf16_f32(kM, D, true);
       uint32_t n_s = 0, n_pv = 0, j = 0;
       int li = 0, s_t = 0, s_nt = 0, s_qb = 0, s_li = 0;
+      uint32_t s_idesc = 0, s_pvdesc = 0;
       bool s_have = false, items_done = false, ok = true;
-      uint8_t tflag[4];  // per issued S tile: bit 0 first tile of its item, bit 1 its last
-      int tli[4];        // item number of the tile (o_empty parity)
+      uint8_t tflag[4];     // per issued S^T tile: bit 0 first tile of its item, bit 1 its last
+      int tli[4];           // item number of the tile (O buffer, o_empty parity)
+      uint32_t tpv[4];      // instruction descriptor of the tile's PV product
       long long last = clock64();
       while (true) {
         bool prog = false;
@@ -355,9 +412,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (it < 0) {
               items_done = true;
             } else {
+              const int nrow = (w.rows + 15) / 16 * 16;  // the MMA's N: rows rounded up to 16
+              s_idesc = ptx::idesc_bf16_f32(kBT, nrow, false, false);
+              s_pvdesc = ptx::idesc_bf16_f32(128, nrow, true, true);
               s_have = true;
               s_t = 0;
-              s_nt = (w.t1 - w.t0 + kBN - 1) / kBN;
+              s_nt = (w.t1 - w.t0 + kBT - 1) / kBT;
               s_qb = li & 1;
               s_li = li;
               ++li;
@@ -366,46 +426,50 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         if (s_have && n_s < n_pv + 4) {
-          const int st = (int)(n_s % C::NSTAGE), sb = n_s & 1;
+          const int st = (int)(n_s % C::NSK), sb = n_s & 1;
           if ((s_t > 0 || ptx::mbar_test_wait(B.q_full + s_qb, (s_li >> 1) & 1)) &&
-              ptx::mbar_test_wait(B.k_full + st, (n_s / C::NSTAGE) & 1) &&
+              ptx::mbar_test_wait(B.k_full + st, (n_s / C::NSK) & 1) &&
               ptx::mbar_test_wait(B.s_empty + sb, ((n_s >> 1) & 1) ^ 1)) {
             ptx::tc_fence_after();
             const uint32_t qa = sbase + C::OFF_Q + s_qb * C::Q_BYTES;
             const uint32_t ka = sbase + C::OFF_K + st * C::KV_TILE;
 #pragma unroll
             for (int ks = 0; ks < D / 16; ++ks) {
-              const uint32_t koff = (ks >> 2) * (kBN * 128) + (ks & 3) * 32;
-              const uint32_t qoff = (ks >> 2) * (kM * 128) + (ks & 3) * 32;
-              ptx::umma_f16(tmem + sb * 64, ptx::sdesc_sw128(qa + qoff, 16, 1024),
-                            ptx::sdesc_sw128(ka + koff, 16, 1024), IDESC_S, ks > 0);
+              const uint32_t koff = (ks >> 2) * C::HALF + (ks & 3) * 32;
+              const uint32_t qoff = (ks >> 2) * C::QHALF + (ks & 3) * 32;
+              ptx::umma_f16(tmem + sb * kNR, ptx::sdesc_sw128(ka + koff, 16, 1024),
+                            ptx::sdesc_sw128(qa + qoff, 16, 1024), s_idesc, ks > 0);
             }
             ptx::umma_commit(B.s_full + sb);
             ptx::umma_commit(B.k_empty + st);
             if (s_t == s_nt - 1) ptx::umma_commit(B.q_empty + s_qb);
             tflag[n_s & 3] = (s_t == 0 ? 1 : 0) | (s_t == s_nt - 1 ? 2 : 0);
             tli[n_s & 3] = s_li;
+            tpv[n_s & 3] = s_pvdesc;
             ++n_s;
             if (++s_t == s_nt) s_have = false;
             prog = true;
           }
         }
         if (n_pv < n_s) {
-          const int pb = (int)(n_pv % 3);
+          const int pb = (int)(n_pv % C::NP);
           const bool first = tflag[n_pv & 3] & 1, last = tflag[n_pv & 3] & 2;
           const int tl = tli[n_pv & 3], ob = tl & 1;  // the item's O buffer
-          const int st = (int)(n_pv % C::NSTAGE);
-          if (ptx::mbar_test_wait(B.p_full + pb, (n_pv / 3) & 1) &&
-              ptx::mbar_test_wait(B.v_full + st, (n_pv / C::NSTAGE) & 1) &&
+          const int st = (int)(n_pv % C::NSV);
+          if (ptx::mbar_test_wait(B.p_full + pb, (n_pv / C::NP) & 1) &&
+              ptx::mbar_test_wait(B.v_full + st, (n_pv / C::NSV) & 1) &&
               (!first || ptx::mbar_test_wait(B.o_empty + ob, ((tl >> 1) & 1) ^ 1))) {
             ptx::tc_fence_after();
             const uint32_t pa = sbase + C::OFF_P + pb * C::P_BYTES;
             const uint32_t va = sbase + C::OFF_V + st * C::KV_TILE;
+            // A = V^T, MN-major: the head dim's 64-wide halves are HALF apart (for D = 64 both MMA
+            // halves read the same half, so O^T lanes 64..127 repeat lanes 0..63 and are not used)
+            constexpr uint32_t lbo_v = D == 128 ? C::HALF : 0;
 #pragma unroll
-            for (int ks = 0; ks < kBN / 16; ++ks) {
-              const uint64_t a = ptx::sdesc_sw128(pa + ks * 32, 16, 1024);
-              const uint64_t b = ptx::sdesc_sw128(va + ks * 16 * 128, kBN * 128, 1024);
-              ptx::umma_f16(tmem + 128 + ob * 128, a, b, IDESC_PV, (!first || ks > 0) ? 1u : 0u);
+            for (int ks = 0; ks < kBT / 16; ++ks) {
+              const uint64_t a = ptx::sdesc_sw128(va + ks * 16 * 128, lbo_v, 1024);
+              const uint64_t b = ptx::sdesc_sw128(pa + ks * 16 * 128, C::P_BYTES, 1024);
+              ptx::umma_f16(tmem + 128 + ob * kNR, a, b, tpv[n_pv & 3], (!first || ks > 0) ? 1u : 0u);
             }
             ptx::umma_commit(B.o_full + pb);
             ptx::umma_commit(B.v_empty + st);
@@ -436,12 +500,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= 8) {
     // ------------------------------------------------------------------ epilogue warps
-    // One warp per TMEM lane quadrant.  Item li's O (buffer li & 1) is read once the softmax warps
-    // have handed the item over and its last PV is done; the output (or, for a split item, the
-    // partial O, m, l) is written, the buffer released, and the last chunk of a split
-    // (request, head) to finish merges all of its chunks.
+    // One warp per TMEM lane quadrant: thread d (lane d of O^T) owns head-dim index d of every row.
+    // Item li's O^T (buffer li & 1) is read once the softmax warps have handed the item over and
+    // its last PV is done; the output (or, for a split item, the partial O, m, l) is written, the
+    // buffer released, and the last chunk of a split (request, head, row group) to finish merges
+    // all of its chunks.
     const int qd = warp & 3;
-    const int mrow = qd * 32 + lane;
+    const int d = qd * 32 + lane;
+    const bool dval = d < D;  // for D = 64 the upper two quadrants hold copies
     const uint32_t lane_addr = (uint32_t)(qd * 32) << 16;
     uint32_t gph = 0;
     int li = 0;
@@ -460,131 +526,127 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(B.it_empty + slot);
       if (it < 0) break;
-      const int G = row_group(w.rows), rep = kM / G;
-      const int rid = (qd * 32) / G;   // replica of this warp's rows
-      const int row = mrow - rid * G;  // query row of this thread (j*g + hh)
-      const int dcw = D / rep;         // this warp writes the output columns [d0, d0 + dcw)
-      const int d0 = rid * dcw;
-      const int jq = row / g;
       const int ob = li & 1;
-      const uint32_t o_col = 128 + ob * 128;
+      const uint32_t o_col = 128 + ob * kNR;
       // the softmax warps' hand-over and the item's last PV
       if (!wait_bar(B.ep_full + ob, (li >> 1) & 1, s_abort)) { ok = false; break; }
       if (!wait_bar(B.o_done + ob, (li >> 1) & 1, s_abort)) { ok = false; break; }
       ++li;
       ptx::tc_fence_after();
-      uint32_t lm[2];
-      ptx::tmem_ld2(tmem + lane_addr + 384 + 2 * ob, lm);
-      ptx::tmem_wait_ld();
-      const float m_ref = __uint_as_float(lm[1]);
-      // row sum: the shares of the row's replicas
-      s_lsum[ob * 128 + mrow] = __uint_as_float(lm[0]);
-      if (!group_sync()) { ok = false; break; }
-      float lt = 0.0f;
-      for (int rr = 0; rr < rep; ++rr) lt += s_lsum[ob * 128 + rr * G + row];
-      const bool ract = row < w.rows;
-      const int hh = row % g;
-      const float inv = 1.0f / lt;
-      for (int c = 0; c < dcw; c += 16) {
-        uint32_t x[16];
-        ptx::tmem_ld16(tmem + lane_addr + o_col + d0 + c, x);
+      const int nc = (w.rows + 31) / 32;
+      for (int c = 0; c < nc; ++c) {
+        uint32_t x[32];  // O^T[d][rows 32c..]
+        ptx::tmem_ld32(tmem + lane_addr + o_col + 32 * c, x);
         ptx::tmem_wait_ld();
-        if (ract) {
-          if (w.poff < 0) {
-            uint16_t *og = static_cast<uint16_t *>(p.out) + ((int64_t)(w.q0 + jq) * p.Hq + w.h * g + hh) * D + d0 + c;
+        // lane i: row 32c + i's sum (the four softmax warps' shares)
+        const int jl = 32 * c + lane;
+        const float *hl = s_hl + ob * 4 * kNR;
+        const float lsum = hl[jl] + hl[kNR + jl] + hl[2 * kNR + jl] + hl[3 * kNR + jl];
+        if (w.poff < 0) {
+          const float linv = 1.0f / lsum;
+          uint16_t *og = static_cast<uint16_t *>(p.out);
 #pragma unroll
-            for (int v = 0; v < 2; ++v) {
-              uint4 o;
-              o.x = pack_bf16(__uint_as_float(x[8 * v + 0]) * inv, __uint_as_float(x[8 * v + 1]) * inv);
-              o.y = pack_bf16(__uint_as_float(x[8 * v + 2]) * inv, __uint_as_float(x[8 * v + 3]) * inv);
-              o.z = pack_bf16(__uint_as_float(x[8 * v + 4]) * inv, __uint_as_float(x[8 * v + 5]) * inv);
-              o.w = pack_bf16(__uint_as_float(x[8 * v + 6]) * inv, __uint_as_float(x[8 * v + 7]) * inv);
-              reinterpret_cast<uint4 *>(og)[v] = o;
+          for (int i = 0; i < 32; ++i) {
+            const int jr = 32 * c + i;
+            const float inv = __shfl_sync(0xffffffffu, linv, i);
+            if (jr < w.rows && dval) {
+              const int rj = w.row0 + jr, jq = rj / g, hh = rj % g;
+              const float o = __uint_as_float(x[i]) * inv;
+              og[((int64_t)(w.q0 + jq) * p.Hq + w.h * g + hh) * D + d] = __bfloat16_as_ushort(__float2bfloat16_rn(o));
             }
-          } else {
-            float4 *part = reinterpret_cast<float4 *>(p.partials + w.poff + (int64_t)row * D + d0 + c);
+          }
+        } else {
+          float *part = p.partials + w.poff;
 #pragma unroll
-            for (int v = 0; v < 4; ++v)
-              part[v] = make_float4(__uint_as_float(x[4 * v]), __uint_as_float(x[4 * v + 1]),
-                                    __uint_as_float(x[4 * v + 2]), __uint_as_float(x[4 * v + 3]));
+          for (int i = 0; i < 32; ++i) {
+            const int jr = 32 * c + i;
+            if (jr < w.rows && dval) __stcg(part + (int64_t)jr * D + d, __uint_as_float(x[i]));
+          }
+          if (qd == 0 && jl < w.rows) {
+            __stcg(part + w.rows * D + jl, s_hm[ob * kNR + jl]);
+            __stcg(part + w.rows * D + w.rows + jl, lsum);
           }
         }
-      }
-      if (ract && rid == 0 && w.poff >= 0) {
-        p.partials[w.poff + w.rows * D + row] = m_ref;
-        p.partials[w.poff + w.rows * D + w.rows + row] = lt;
       }
       ptx::tc_fence_before();
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(B.o_empty + ob);
 
-      // ---- split item: the last chunk of this (request, head) to finish merges all chunks ----
+      // ---- split item: the last chunk of this (request, head, row group) to finish merges all ----
       if (w.poff >= 0) {
         __threadfence();
         if (!group_sync()) { ok = false; break; }
         if (warp == 8 && lane == 0) {
           const int chunks = p.req_chunks[w.r];
-          const int done = atomicAdd(p.pair_done + (int64_t)w.r * p.Hkv + w.h, 1);
+          const int done = atomicAdd(p.pair_done + ((int64_t)w.r * p.Hkv + w.h) * 2 + w.rg, 1);
           *s_last = done == chunks - 1 ? chunks : 0;
           __threadfence();
         }
         if (!group_sync()) { ok = false; break; }
         const int chunks = *s_last;
-        if (chunks > 0 && ract) {
-          // every warp merges its column slice of its rows
-          const WorkItem *ci = p.items + p.req_item_begin[w.r] + w.h * chunks;
-          float mstar = -INFINITY;
-          for (int c = 0; c < chunks; ++c)
-            mstar = fmaxf(mstar, __ldcg(p.partials + ci[c].poff + w.rows * D + row));
-          float den = 0.0f;
-          for (int c = 0; c < chunks; ++c) {
-            const float *part = p.partials + ci[c].poff;
-            const float mc = __ldcg(part + w.rows * D + row);
-            if (mc != -INFINITY) den = fmaf(__ldcg(part + w.rows * D + w.rows + row), ptx::ex2(mc - mstar), den);
-          }
-          const float dinv = 1.0f / den;
-          uint16_t *og = static_cast<uint16_t *>(p.out) + ((int64_t)(w.q0 + jq) * p.Hq + w.h * g + hh) * D;
-          for (int d = d0; d < d0 + dcw; d += 16) {
-            float acc[16];
-#pragma unroll
-            for (int i = 0; i < 16; ++i) acc[i] = 0.0f;
+        if (chunks > 0) {
+          const WorkItem *ci = p.items + p.req_item_begin[w.r] + (w.h * w.nrg + w.rg) * chunks;
+          // thread jr < rows: row jr's overall max and 1 / sum over the chunks
+          if (d < w.rows) {
+            float mstar = -INFINITY;
+            for (int c = 0; c < chunks; ++c) mstar = fmaxf(mstar, __ldcg(p.partials + ci[c].poff + w.rows * D + d));
+            float den = 0.0f;
             for (int c = 0; c < chunks; ++c) {
               const float *part = p.partials + ci[c].poff;
-              const float mc = __ldcg(part + w.rows * D + row);
-              if (mc == -INFINITY) continue;
-              const float wgt = ptx::ex2(mc - mstar);
-              const float4 *src = reinterpret_cast<const float4 *>(part + (int64_t)row * D + d);
+              const float mc = __ldcg(part + w.rows * D + d);
+              if (mc != -INFINITY) den = fmaf(__ldcg(part + w.rows * D + w.rows + d), ptx::ex2(mc - mstar), den);
+            }
+            s_em[d] = mstar;
+            s_em[kNR + d] = 1.0f / den;
+          }
+          if (!group_sync()) { ok = false; break; }
+          // thread d: column d of every row, eight rows at a time (independent loads in flight)
+          if (dval) {
+            uint16_t *og = static_cast<uint16_t *>(p.out);
+            for (int j0 = 0; j0 < w.rows; j0 += 8) {
+              float acc[8];
 #pragma unroll
-              for (int v = 0; v < 4; ++v) {
-                const float4 a = __ldcg(src + v);
-                acc[4 * v] = fmaf(a.x, wgt, acc[4 * v]);
-                acc[4 * v + 1] = fmaf(a.y, wgt, acc[4 * v + 1]);
-                acc[4 * v + 2] = fmaf(a.z, wgt, acc[4 * v + 2]);
-                acc[4 * v + 3] = fmaf(a.w, wgt, acc[4 * v + 3]);
+              for (int q = 0; q < 8; ++q) acc[q] = 0.0f;
+#pragma unroll 4
+              for (int c = 0; c < chunks; ++c) {
+                const float *part = p.partials + ci[c].poff;
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                  const int jr = j0 + q;
+                  if (jr < w.rows) {
+                    const float mc = __ldcg(part + w.rows * D + jr);
+                    const float ov = __ldcg(part + (int64_t)jr * D + d);
+                    if (mc != -INFINITY) acc[q] = fmaf(ov, ptx::ex2(mc - s_em[jr]), acc[q]);
+                  }
+                }
+              }
+#pragma unroll
+              for (int q = 0; q < 8; ++q) {
+                const int jr = j0 + q;
+                if (jr < w.rows) {
+                  const int rj = w.row0 + jr, jq = rj / g, hh = rj % g;
+                  og[((int64_t)(w.q0 + jq) * p.Hq + w.h * g + hh) * D + d] =
+                      __bfloat16_as_ushort(__float2bfloat16_rn(acc[q] * s_em[kNR + jr]));
+                }
               }
             }
-#pragma unroll
-            for (int v = 0; v < 2; ++v) {
-              uint4 o;
-              o.x = pack_bf16(acc[8 * v + 0] * dinv, acc[8 * v + 1] * dinv);
-              o.y = pack_bf16(acc[8 * v + 2] * dinv, acc[8 * v + 3] * dinv);
-              o.z = pack_bf16(acc[8 * v + 4] * dinv, acc[8 * v + 5] * dinv);
-              o.w = pack_bf16(acc[8 * v + 6] * dinv, acc[8 * v + 7] * dinv);
-              reinterpret_cast<uint4 *>(og + d)[v] = o;
-            }
           }
+          // s_em is read above until every warp is past this point
+          if (!group_sync()) { ok = false; break; }
         }
       }
     }
     if (!ok && lane == 0) report(p.status, WISP_DEV_TIMEOUT, p.request_ids, 0);
   } else {
     // ------------------------------------------------------------------ softmax warps
-    const int qd = warp & 3;          // TMEM lane quadrant of this warp
-    const int mrow = qd * 32 + lane;  // this thread's MMA row
+    const int qd = warp & 3;          // TMEM lane quadrant of this warp: keys 32*qd .. 32*qd + 31 of a tile
     const uint32_t lane_addr = (uint32_t)(qd * 32) << 16;
     const float scale_log2 = 1.4426950408889634f / sqrtf((float)D);
-    uint32_t n = 0;
-    int li = 0;  // items so far: item li accumulates into O buffer li & 1
+    float *mw = s_mw + qd * kNR;      // this warp's copy of the rows' reference maxima
+    float *fw = s_fw + qd * kNR;      // this warp's copy of the rescale factors
+    float *tr = s_tr + qd * 32 * 33;  // this warp's transpose scratch
+    uint32_t n = 0, nf = 0;           // tiles so far; tiles that moved a reference max
+    int li = 0;                       // items so far: item li accumulates into O buffer li & 1
     bool ok = true;
     for (uint32_t j = 0; ok; ++j) {
       const int slot = j % C::RING;
@@ -594,178 +656,225 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(B.it_empty + slot);
       if (it < 0) break;
-      const int G = row_group(w.rows), rep = kM / G;
-      const int rid = (qd * 32) / G;      // replica handled by this warp
-      const int row = mrow - rid * G;     // query row of this thread (j*g + hh)
-      const int cw = kBN / rep;           // columns of each S tile handled by this warp
-      const int c0 = rid * cw;
-      // P is written to every replica row, so O = P V comes out replicated in all four lane
-      // quadrants; this warp rescales the O columns [d0, d0 + dcw) of its quadrant
-      const int dcw = D / rep;
-      const int d0 = rid * dcw;
-      const int jq = row / g;
-      const int vis = w.ctx + jq;         // last key position this row may see
       const int ob = li & 1;
-      const uint32_t o_col = 128 + ob * 128;
-      float m_ref = -INFINITY, l = 0.0f;
+      const uint32_t o_col = 128 + ob * kNR;
+      const int ntiles = (w.t1 - w.t0 + kBT - 1) / kBT;
+      const int nu = (w.rows + 15) / 16 * 2;  // 8-row units the MMA reads (its N / 8)
+      mw[lane] = -INFINITY;
+      mw[lane + 32] = -INFINITY;
+      __syncwarp();
 
-      const int ntiles = (w.t1 - w.t0 + kBN - 1) / kBN;
-      // the tile loop, specialised for the CW columns of each S tile this warp handles
-      auto run_tiles = [&](auto cw_tag) -> bool {
-        constexpr int CW = decltype(cw_tag)::value;
+      // the tile loop, specialised for the 32-row chunks of the item
+      auto run_tiles = [&](auto nc_tag) -> bool {
+        constexpr int NC = decltype(nc_tag)::value;
+        float lp[NC][32];  // this thread's (key's) share of every row sum
+#pragma unroll
+        for (int c = 0; c < NC; ++c)
+#pragma unroll
+          for (int i = 0; i < 32; ++i) lp[c][i] = 0.0f;
         for (int t = 0; t < ntiles; ++t, ++n) {
           const int sb = n & 1;
           if (!wait_bar(B.s_full + sb, (n >> 1) & 1, s_abort)) return false;
           ptx::tc_fence_after();
-          // the whole 64-column row (replicas hold identical rows, so each warp gets the row max
-          // without talking to the others), then this warp's CW columns
-          float sr[kBN];
+          // P buffer n % NP is free again once PV(n - NP) is done (this thread waited PV(n - 2NP)
+          // before, and PV(n) needs the P(n) it is about to publish: the parity is exact)
+          const int pbuf = (int)(n % C::NP);
+          if (n >= (uint32_t)C::NP && !wait_bar(B.o_full + pbuf, ((n - C::NP) / C::NP) & 1, s_abort)) return false;
+          // this key's row of P^T: 128 bytes (64 rows, bf16), 16-byte units swizzled by key & 7
+          uint8_t *prow = smem + C::OFF_P + pbuf * C::P_BYTES + (qd * 32 + lane) * 128;
+          const int sw = lane & 7;
+          // causal mask: key tok is visible to row jr iff tok <= ctx + (row0 + jr) / g, i.e.
+          // row0 + jr >= g * (tok - ctx); keys past the item and rows past `rows` are masked too
+          const int tok = w.t0 + t * kBT + qd * 32 + lane;
+          const int jmin = tok >= w.t1 ? kNR : max(0, g * (tok - w.ctx) - w.row0);
+          const int jmax = w.rows;
+          // P = 2^(s - m) against the current reference maxima (masked: 0), written straight to the
+          // P buffer and added to the row-sum shares; the vote asks whether any P exceeds 2^kTau
+          // (then the tile is redone below with new references)
+          float emax = 0.0f;
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
+          for (int c = 0; c < NC; ++c) {
             uint32_t x[32];
-            ptx::tmem_ld32(tmem + lane_addr + sb * 64 + h * 32, x);
+            ptx::tmem_ld32(tmem + lane_addr + sb * kNR + 32 * c, x);
             ptx::tmem_wait_ld();
 #pragma unroll
-            for (int i = 0; i < 32; ++i) sr[h * 32 + i] = __uint_as_float(x[i]);
-          }
-
-          const int tok0 = w.t0 + t * kBN;
-          // interior tile: every token visible to every row of the item
-          const bool interior = tok0 + kBN <= w.t1 && tok0 + kBN - 1 <= w.ctx;
-          if (!interior) {
+            for (int u = 0; u < 4; ++u) {
+              if (4 * c + u < nu) {
+                uint32_t pk[4];
 #pragma unroll
-            for (int i = 0; i < kBN; ++i) {
-              const int tok = tok0 + i;
-              if (!(tok < w.t1 && tok <= vis)) sr[i] = -INFINITY;
+                for (int h = 0; h < 2; ++h) {
+                  const int i0 = 8 * u + 4 * h;
+                  const float4 m4 = reinterpret_cast<const float4 *>(mw + 32 * c + i0)[0];
+                  const float mm[4] = {m4.x, m4.y, m4.z, m4.w};
+                  float e[4];
+#pragma unroll
+                  for (int q = 0; q < 4; ++q) {
+                    const int jr = 32 * c + i0 + q;
+                    const float v = ptx::ex2(fmaf(__uint_as_float(x[i0 + q]), scale_log2, -mm[q]));
+                    e[q] = (jr >= jmin && jr < jmax) ? v : 0.0f;
+                    emax = fmaxf(emax, e[q]);
+                    lp[c][i0 + q] += e[q];
+                  }
+                  pk[2 * h] = pack_bf16(e[0], e[1]);
+                  pk[2 * h + 1] = pack_bf16(e[2], e[3]);
+                }
+                *reinterpret_cast<uint4 *>(prow + (((4 * c + u) ^ sw) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+              }
             }
           }
-          // row max with eight independent partial maxima (short dependency chains)
-          float m8[8];
-#pragma unroll
-          for (int k = 0; k < 8; ++k) m8[k] = sr[k];
-#pragma unroll
-          for (int i = 8; i < kBN; ++i) m8[i & 7] = fmaxf(m8[i & 7], sr[i]);
-#pragma unroll
-          for (int k = 0; k < 4; ++k) m8[k] = fmaxf(m8[k], m8[k + 4]);
-          const float m_tile = fmaxf(fmaxf(m8[0], m8[2]), fmaxf(m8[1], m8[3])) * scale_log2;  // scale > 0
-          float sv[CW];
-          if constexpr (CW == kBN) {
-#pragma unroll
-            for (int i = 0; i < CW; ++i) sv[i] = sr[i] * scale_log2;  // -inf stays -inf
-          } else {
-            // this warp's own CW columns, taken from the (already masked) row in registers; the
-            // replica index is warp-uniform, so each case reads registers at constant indices
-            auto take = [&](auto part) {
-              constexpr int o = decltype(part)::value * CW;
-#pragma unroll
-              for (int i = 0; i < CW; ++i) sv[i] = sr[o + i] * scale_log2;
-            };
-            const int part = c0 / CW;
-            if (part == 0) take(std::integral_constant<int, 0>{});
-            else if (part == 1) take(std::integral_constant<int, 1>{});
-            if constexpr (CW == 16) {
-              if (part == 2) take(std::integral_constant<int, 2>{});
-              else if (part == 3) take(std::integral_constant<int, 3>{});
-            }
+          // the four warps' votes, double-buffered by tile parity (NaN never wins fmaxf, and a
+          // visible key of a row without a reference yet gives +inf)
+          const uint32_t vote = __ballot_sync(0xffffffffu, !(emax <= kExpTau));
+          if (lane == 0) {
+            s_flag[(n & 1) * 4 + qd] = vote;
+            ptx::mbar_arrive(B.sm_sync);
           }
-          // S(n) has been read: its TMEM buffer may be overwritten by S(n+2)
-          ptx::tc_fence_before();
-          __syncwarp();
-          if (lane == 0) ptx::mbar_arrive(B.s_empty + sb);
-          float fac = 1.0f;
-          bool rescale = false;
-          if (m_ref == -INFINITY) {
-            m_ref = m_tile;  // O holds nothing for this row yet
-          } else if (m_tile > m_ref + kTau) {
-            fac = ptx::ex2(m_ref - m_tile);
-            rescale = true;
-            m_ref = m_tile;
-          }
-          const float m_use = m_ref == -INFINITY ? 0.0f : m_ref;
-          l *= fac;
-          uint32_t pk[CW / 2];
-          float ev[CW];
+          if (!wait_bar(B.sm_sync, n & 1, s_abort)) return false;
+          const bool any = (s_flag[(n & 1) * 4] | s_flag[(n & 1) * 4 + 1] | s_flag[(n & 1) * 4 + 2] |
+                            s_flag[(n & 1) * 4 + 3]) != 0;
+          if (any) {
+            // new references: exact tile maxima per row (over this warp's 32 keys through the
+            // transpose scratch, then over the four warps), from the scores read again
 #pragma unroll
-          for (int i = 0; i < CW; ++i) ev[i] = ptx::ex2(sv[i] - m_use);
-#pragma unroll
-          for (int i = 0; i < CW; i += 2) pk[i / 2] = pack_bf16(ev[i], ev[i + 1]);
-#pragma unroll
-          for (int w2 = 1; w2 < CW; w2 <<= 1) {
-#pragma unroll
-            for (int i = 0; i < CW; i += 2 * w2) ev[i] += ev[i + w2];
-          }
-          l += ev[0];
-          // PV(m) completes barrier o_full[m % 3] for the (m / 3)-th time.  Every softmax warp
-          // waits PV(n-3) here (P buffer n % 3 is free again); since it waited PV(n-6) three tiles
-          // ago and PV(n) needs the P(n) it is about to publish, the parity names exactly PV(n-3).
-          const int pbuf = (int)(n % 3);
-          if (n >= 3 && !wait_bar(B.o_full + pbuf, ((n - 3) / 3) & 1, s_abort)) return false;
-          // a rescale of the O rows needs PV(n-1) complete (exact for the same reason) and
-          // precedes PV(n); each warp rescales its own column slice of its quadrant's rows
-          if (t > 0 && __ballot_sync(0xffffffffu, rescale)) {
-            if (!wait_bar(B.o_full + (n - 1) % 3, ((n - 1) / 3) & 1, s_abort)) return false;
-            ptx::tc_fence_after();
-            for (int c = 0; c < dcw; c += 16) {
-              uint32_t x[16];
-              ptx::tmem_ld16(tmem + lane_addr + o_col + d0 + c, x);
+            for (int c = 0; c < NC; ++c) {
+              uint32_t x[32];
+              ptx::tmem_ld32(tmem + lane_addr + sb * kNR + 32 * c, x);
               ptx::tmem_wait_ld();
 #pragma unroll
-              for (int i = 0; i < 16; ++i) x[i] = __float_as_uint(__uint_as_float(x[i]) * fac);
-              ptx::tmem_st16(tmem + lane_addr + o_col + d0 + c, x);
-            }
-            ptx::tmem_wait_st();
-            ptx::tc_fence_before();
-          }
-          // this warp's columns of P row `row` (bf16, 128-byte swizzle)
+              for (int i = 0; i < 32; ++i) {
+                const int jr = 32 * c + i;
+                tr[lane * 33 + i] = (jr >= jmin && jr < jmax) ? __uint_as_float(x[i]) * scale_log2 : -INFINITY;  // scale > 0
+              }
+              __syncwarp();
+              float tm = -INFINITY;
 #pragma unroll
-          for (int rr = 0; rr < kBN / CW; ++rr) {
-            uint8_t *prow = smem + C::OFF_P + pbuf * C::P_BYTES + (rr * G + row) * 128;  // (rr*G + row) & 7 == row & 7
+              for (int i = 0; i < 32; ++i) tm = fmaxf(tm, tr[i * 33 + lane]);
+              s_red[qd * kNR + 32 * c + lane] = tm;
+              __syncwarp();
+            }
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(B.sm_sync2);
+            if (!wait_bar(B.sm_sync2, nf & 1, s_abort)) return false;
+            ++nf;
+            // take this tile's P back out of the shares (a row without a reference had nothing yet)
 #pragma unroll
-            for (int c = 0; c < CW / 8; ++c) {
-              const int cc = c0 / 8 + c;
-              *reinterpret_cast<uint4 *>(prow + ((cc ^ (row & 7)) << 4)) =
-                  make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+            for (int c = 0; c < NC; ++c) {
+              uint32_t x[32];
+              ptx::tmem_ld32(tmem + lane_addr + sb * kNR + 32 * c, x);
+              ptx::tmem_wait_ld();
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                const int jr = 32 * c + i;
+                const float mo = mw[jr];
+                const float v = ptx::ex2(fmaf(__uint_as_float(x[i]), scale_log2, -mo));
+                const float eo = (jr >= jmin && jr < jmax) ? v : 0.0f;
+                lp[c][i] = mo == -INFINITY ? 0.0f : lp[c][i] - eo;
+              }
+            }
+            __syncwarp();
+            // every warp derives the same new maxima and factors from the same values
+            bool moved = false;
+#pragma unroll
+            for (int c = 0; c < NC; ++c) {
+              const int jl = 32 * c + lane;
+              const float tmax = fmaxf(fmaxf(s_red[jl], s_red[kNR + jl]), fmaxf(s_red[2 * kNR + jl], s_red[3 * kNR + jl]));
+              const float mo = mw[jl];
+              const float mn = tmax > mo + kTau ? tmax : mo;
+              fw[jl] = mn == mo ? 1.0f : (mo == -INFINITY ? 0.0f : ptx::ex2(mo - mn));
+              moved |= mn != mo && mo != -INFINITY;
+              mw[jl] = mn;
+            }
+            __syncwarp();
+            // P again against the new references: shares rescaled, P rewritten
+#pragma unroll
+            for (int c = 0; c < NC; ++c) {
+              uint32_t x[32];
+              ptx::tmem_ld32(tmem + lane_addr + sb * kNR + 32 * c, x);
+              ptx::tmem_wait_ld();
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                uint32_t pk[4];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                  float e[4];
+#pragma unroll
+                  for (int q = 0; q < 4; ++q) {
+                    const int i = 8 * u + 4 * h + q, jr = 32 * c + i;
+                    const float v = ptx::ex2(fmaf(__uint_as_float(x[i]), scale_log2, -mw[jr]));
+                    e[q] = (jr >= jmin && jr < jmax) ? v : 0.0f;
+                    lp[c][i] = fmaf(lp[c][i], fw[jr], e[q]);
+                  }
+                  pk[2 * h] = pack_bf16(e[0], e[1]);
+                  pk[2 * h + 1] = pack_bf16(e[2], e[3]);
+                }
+                if (4 * c + u < nu)
+                  *reinterpret_cast<uint4 *>(prow + (((4 * c + u) ^ sw) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+              }
+            }
+            // O^T, if it holds earlier tiles of the item, moves to the new references; the rescale
+            // needs PV(n-1) complete and precedes PV(n)
+            if (t > 0 && __any_sync(0xffffffffu, moved)) {
+              // PV(m) completes barrier o_full[m % NP] for the (m / NP)-th time; this thread has
+              // waited PV(n-NP) already and PV(n-1+NP) needs P(n-1+NP), so the parity names PV(n-1)
+              if (!wait_bar(B.o_full + (n - 1) % C::NP, ((n - 1) / C::NP) & 1, s_abort)) return false;
+              ptx::tc_fence_after();
+#pragma unroll
+              for (int c = 0; c < 2 * NC; ++c) {
+                uint32_t y[16];
+                ptx::tmem_ld16(tmem + lane_addr + o_col + 16 * c, y);
+                ptx::tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 16; ++i) y[i] = __float_as_uint(__uint_as_float(y[i]) * fw[16 * c + i]);
+                ptx::tmem_st16(tmem + lane_addr + o_col + 16 * c, y);
+              }
+              ptx::tmem_wait_st();
             }
           }
+          // S^T(n) has been read: its TMEM buffer may be overwritten by S^T(n+2); P(n) is published
+          ptx::tc_fence_before();
           ptx::fence_proxy_async_smem();
           __syncwarp();
-          if (lane == 0) ptx::mbar_arrive(B.p_full + pbuf);
+          if (lane == 0) {
+            ptx::mbar_arrive(B.s_empty + sb);
+            ptx::mbar_arrive(B.p_full + pbuf);
+          }
         }
+        // ---- hand the item over to the epilogue warps: this warp's share of each row sum and the
+        // reference maxima.  The epilogue of item li - 2 (same buffers) must be done with them.
+        float lsh[NC];
+#pragma unroll
+        for (int c = 0; c < NC; ++c) lsh[c] = warp_transpose_reduce<false>(lp[c], tr, lane);
+        if (!wait_bar(B.o_empty + ob, ((li >> 1) & 1) ^ 1, s_abort)) return false;
+#pragma unroll
+        for (int c = 0; c < NC; ++c) {
+          s_hl[(ob * 4 + qd) * kNR + 32 * c + lane] = lsh[c];
+          if (qd == 0) s_hm[ob * kNR + 32 * c + lane] = mw[32 * c + lane];
+        }
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(B.ep_full + ob);
         return true;
       };
-      if (cw == 16) {
-        ok = run_tiles(std::integral_constant<int, 16>{});
-      } else if (cw == 32) {
-        ok = run_tiles(std::integral_constant<int, 32>{});
+      if (w.rows <= 32) {
+        ok = run_tiles(std::integral_constant<int, 1>{});
       } else {
-        ok = run_tiles(std::integral_constant<int, 64>{});
+        ok = run_tiles(std::integral_constant<int, 2>{});
       }
       if (!ok) break;
-
-      // ---- hand the item over to the epilogue warps: this thread's share of the row sum and the
-      // reference max go to two spare TMEM columns of its lane.  The epilogue of item li - 2 (same
-      // O buffer and columns) must be done with them first.
-      if (!wait_bar(B.o_empty + ob, ((li >> 1) & 1) ^ 1, s_abort)) { ok = false; break; }
-      ptx::tc_fence_after();
-      {
-        const uint32_t lm[2] = {__float_as_uint(l), __float_as_uint(m_ref)};
-        ptx::tmem_st2(tmem + lane_addr + 384 + 2 * ob, lm);
-        ptx::tmem_wait_st();
-      }
-      ptx::tc_fence_before();
-      __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(B.ep_full + ob);
       ++li;
     }
     if (!ok && lane == 0) report(p.status, WISP_DEV_TIMEOUT, p.request_ids, 0);
   }
 
-  // __syncthreads is an aligned barrier: each warp must reach it converged, and the roles above
-  // leave lane 0 alone in its loop (MMA issue, drains)
+  // Teardown: every warp reports on an mbarrier that it is done with TMEM, and warp 1 frees the
+  // TMEM once all have (a bounded wait; the warps' shared memory stays until the last one exits).
   __syncwarp();
   ptx::tc_fence_before();
-  __syncthreads();
+  if (lane == 0) ptx::mbar_arrive(B.fin);
   if (warp == 1) {
+    const long long t0 = clock64();
+    while (!ptx::mbar_try_wait(B.fin, 0) && clock64() - t0 < kWaitCycles) {
+    }
+    __syncwarp();
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, kTmemCols);
   }
@@ -788,7 +897,7 @@ cudaError_t get_encode() {
 
 // The paged pool [num_blocks, Hkv, 16, D] bf16 as a 4-D tensor (d, slot, head, block);
 // one box = 64 head-dim elements (128 bytes, swizzled) x 16 slots of one head in `box_blocks`
-// consecutive blocks (1, or 4 for a whole 64-token tile of consecutive blocks).
+// consecutive blocks (1, or 8 for a whole 128-token tile of consecutive blocks).
 cudaError_t encode_pool(CUtensorMap *map, const void *base, int D, int Hkv, int num_blocks, int box_blocks) {
   const cuuint64_t dims[4] = {(cuuint64_t)D, 16, (cuuint64_t)Hkv, (cuuint64_t)num_blocks};
   const cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)16 * D * 2, (cuuint64_t)Hkv * 16 * D * 2};
@@ -816,16 +925,16 @@ cudaError_t attn_tc_setup() {
 }
 
 cudaError_t attn_tc_launch(const AttnParams &p, int grid, cudaStream_t s) {
-  alignas(64) CUtensorMap tk, tv, tk4, tv4;
+  alignas(64) CUtensorMap tk, tv, tk8, tv8;
   cudaError_t e = encode_pool(&tk, p.k_cache, p.D, p.Hkv, p.num_blocks, 1);
   if (e == cudaSuccess) e = encode_pool(&tv, p.v_cache, p.D, p.Hkv, p.num_blocks, 1);
-  if (e == cudaSuccess) e = encode_pool(&tk4, p.k_cache, p.D, p.Hkv, p.num_blocks, 4);
-  if (e == cudaSuccess) e = encode_pool(&tv4, p.v_cache, p.D, p.Hkv, p.num_blocks, 4);
+  if (e == cudaSuccess) e = encode_pool(&tk8, p.k_cache, p.D, p.Hkv, p.num_blocks, 8);
+  if (e == cudaSuccess) e = encode_pool(&tv8, p.v_cache, p.D, p.Hkv, p.num_blocks, 8);
   if (e != cudaSuccess) return e;
   if (p.D == 128) {
-    attn_tc_kernel<128><<<grid, kThreads, Cfg<128>::SMEM, s>>>(p, tk, tv, tk4, tv4);
+    attn_tc_kernel<128><<<grid, kThreads, Cfg<128>::SMEM, s>>>(p, tk, tv, tk8, tv8);
   } else {
-    attn_tc_kernel<64><<<grid, kThreads, Cfg<64>::SMEM, s>>>(p, tk, tv, tk4, tv4);
+    attn_tc_kernel<64><<<grid, kThreads, Cfg<64>::SMEM, s>>>(p, tk, tv, tk8, tv8);
   }
   return cudaGetLastError();
 }

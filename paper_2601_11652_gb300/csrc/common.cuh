@@ -25,7 +25,8 @@ __device__ __forceinline__ void report(DeviceStatus *st, int32_t code, const int
   }
 }
 
-constexpr int kMaxRowsPerHead = 128;  // (Hq/Hkv) * (k+1) rows per KV head per work item
+constexpr int kMaxRowsPerHead = 128;  // (Hq/Hkv) * (k+1) rows per KV head of a request
+constexpr int kTcRowsPerItem = 64;    // query rows per work item of the tensor-core attention kernel
 constexpr int kMaxDraft = 1024;       // k_r limit of the acceptance kernels
 
 // Hardware 2^x (ex2.approx.ftz.f32).  Over every float x in [-126, 0] its relative error is below

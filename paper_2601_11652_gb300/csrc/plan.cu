@@ -4,8 +4,9 @@
 // rows and c_r + k_r + 1 keys (L_total = L_cached + L_new, Sec. 4.4).  Lengths
 // live on the device, so the planner runs there: it prefix-sums the row offsets,
 // flags invalid requests, and cuts every (request, KV head) sequence into chunks
-// of at most `chunk_len` keys so that the attention grid has about
-// kItemsPerSM items per SM whatever the length mix.
+// of at most `chunk_len` keys so that the attention grid has about one item per
+// SM (kItemsPerSM when there are fewer (request, head) pairs than SMs) whatever
+// the length mix.
 #include "plan.cuh"
 
 namespace wisp {
@@ -52,7 +53,7 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
   const int64_t cap_tokens = (int64_t)p.max_blocks_per_seq * p.block_size;
 
   // pass 1: offsets (negative lengths count as 0) and validation
-  int64_t carry_q = 0, carry_d = 0, carry_n = 0;
+  int64_t carry_q = 0, carry_d = 0, carry_n = 0, carry_v = 0;
   for (int base = 0; base < p.B; base += kThreads) {
     const int r = base + tid;
     int64_t k = 0, n = 0;
@@ -73,6 +74,8 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     const int64_t id = block_scan(r < p.B ? k : 0, s_warp, &td);
     const int64_t in = block_scan(n, s_warp, &tn);
     (void)in;
+    int64_t tv;
+    (void)block_scan(n > 0 ? 1 : 0, s_warp, &tv);
     if (r < p.B) {
       const int64_t q0 = carry_q + iq - (k + 1), d0 = carry_d + id - k;
       // a request whose rows fall outside the caller's buffers is never touched
@@ -86,6 +89,7 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     carry_q += tq;
     carry_d += td;
     carry_n += tn;
+    carry_v += tv;
   }
   if (tid == 0) {
     p.q_row_start[p.B] = (int32_t)min64(carry_q, INT32_MAX);
@@ -98,26 +102,34 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
   if (!p.with_attention) return;
   __syncthreads();
 
-  // pass 2: chunk length so that sum over (r, h) of ceil(n_r / chunk_len) is about target_items
+  // pass 2: chunk length so that sum over (r, h) of ceil(n_r / chunk_len) is about the item goal:
+  // one item per SM when there are at least as many (request, head) pairs as SMs (a longest-first
+  // order then balances whole sequences and few need the merge of split chunks), else
+  // kItemsPerSM items per SM
   const int64_t work = carry_n * p.Hkv;
-  int64_t chunk = (work + p.target_items - 1) / max(1, p.target_items);
+  const int64_t sms = max(1, p.target_items / kItemsPerSM);
+  const int64_t goal = carry_v * p.Hkv >= sms ? sms : (int64_t)p.target_items;
+  int64_t chunk = (work + goal - 1) / goal;
   chunk = max64(chunk, kMinChunk);
   chunk = (chunk + kChunkAlign - 1) / kChunkAlign * kChunkAlign;
 
-  // pass 3: items and partial slots (request-major, then KV head, then chunk)
+  // pass 3: items and partial slots (request-major, then KV head, then row group, then chunk)
   int64_t item_carry = 0, poff_carry = 0;
   for (int base = 0; base < p.B; base += kThreads) {
     const int r = base + tid;
-    int64_t n = 0, chunks = 0, rows = 0;
+    int64_t n = 0, chunks = 0, rows = 0, nrg = 1, rows0 = 0;
     if (r < p.B && p.req_flag[r] == REQ_OK) {
       n = (int64_t)p.context_lens[r] + p.draft_lens[r] + 1;
       chunks = (n + chunk - 1) / chunk;
       rows = (int64_t)g * (p.draft_lens[r] + 1);
+      nrg = rows > p.max_rows_item ? 2 : 1;
+      rows0 = (rows + nrg - 1) / nrg;  // rows <= 2 * max_rows_item: both groups fit
     }
-    const int64_t nitems = chunks * p.Hkv;
+    const int64_t nitems = chunks * p.Hkv * nrg;
     // each split item's partials start on a 16-byte boundary (vector stores)
-    const int64_t slot = (rows * (p.D + 2) + 3) / 4 * 4;
-    const int64_t pfl = chunks > 1 ? nitems * slot : 0;
+    const int64_t slot_a = (rows0 * (p.D + 2) + 3) / 4 * 4;
+    const int64_t slot_b = nrg == 2 ? ((rows - rows0) * (p.D + 2) + 3) / 4 * 4 : 0;
+    const int64_t pfl = chunks > 1 ? chunks * p.Hkv * (slot_a + slot_b) : 0;
     int64_t ti, tp;
     const int64_t ii = block_scan(nitems, s_warp, &ti);
     const int64_t ip = block_scan(pfl, s_warp, &tp);
@@ -131,21 +143,26 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
         report(p.status, WISP_DEV_UNSUPPORTED, p.request_ids, r);
       }
       p.req_item_begin[r] = (int32_t)first;
-      for (int h = 0; h < p.Hkv; ++h) p.pair_done[(int64_t)r * p.Hkv + h] = 0;
+      for (int h = 0; h < 2 * p.Hkv; ++h) p.pair_done[(int64_t)r * p.Hkv * 2 + h] = 0;
       p.req_chunks[r] = fits ? (int32_t)chunks : 0;
       if (fits) {
         for (int64_t h = 0; h < p.Hkv; ++h) {
-          for (int64_t c = 0; c < chunks; ++c) {
-            WorkItem it;
-            it.r = r;
-            it.h = (int32_t)h;
-            it.t0 = (int32_t)(c * chunk);
-            it.t1 = (int32_t)min64(n, (c + 1) * chunk);
-            it.rows = (int32_t)rows;
-            it.poff = chunks > 1 ? (int32_t)(pfirst + (h * chunks + c) * slot) : -1;
-            it.q0 = p.q_row_start[r];
-            it.ctx = p.context_lens[r];
-            p.items[first + h * chunks + c] = it;
+          for (int64_t rg = 0; rg < nrg; ++rg) {
+            for (int64_t c = 0; c < chunks; ++c) {
+              WorkItem it;
+              it.r = r;
+              it.h = (int32_t)h;
+              it.t0 = (int32_t)(c * chunk);
+              it.t1 = (int32_t)min64(n, (c + 1) * chunk);
+              it.row0 = rg ? (int32_t)rows0 : 0;
+              it.rows = (int32_t)(rg ? rows - rows0 : rows0);
+              it.rg = (int32_t)rg;
+              it.nrg = (int32_t)nrg;
+              it.poff = chunks > 1 ? (int32_t)(pfirst + (h * chunks + c) * (slot_a + slot_b) + (rg ? slot_a : 0)) : -1;
+              it.q0 = p.q_row_start[r];
+              it.ctx = p.context_lens[r];
+              p.items[first + (h * nrg + rg) * chunks + c] = it;
+            }
           }
         }
       }

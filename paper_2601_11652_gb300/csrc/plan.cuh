@@ -5,13 +5,19 @@
 
 namespace wisp {
 
-// One unit of attention work: KV tokens [t0, t1) of request r for KV head h.
+// One unit of attention work: KV tokens [t0, t1) of request r for KV head h, query rows
+// [row0, row0 + rows) of the (Hq/Hkv) * (k_r + 1) rows of that head (row = j * (Hq/Hkv) + hh for
+// query position j and head hh of the group).  The row set of a (request, head) is cut into
+// nrg groups when it is larger than the kernel's row limit.
 struct WorkItem {
   int32_t r, h, t0, t1;
   int32_t poff;   // offset (floats) of this item's split partials, -1 if the item covers the whole sequence
-  int32_t rows;   // query rows of the item: (Hq/Hkv) * (k_r + 1)
+  int32_t rows;   // query rows of the item
   int32_t q0;     // first query row of request r
   int32_t ctx;    // c_r
+  int32_t row0;   // first query row of the item within its (request, head)
+  int32_t rg;     // row group of the item
+  int32_t nrg;    // row groups of its (request, head): 1 or 2
 };
 
 struct PlanHeader {
@@ -22,7 +28,8 @@ struct PlanHeader {
   int32_t pad[4];
 };
 
-constexpr int kItemsPerSM = 2;     // target work items per SM for split-KV (measured best of 1, 2, 4, 6, 8)
+constexpr int kItemsPerSM = 2;     // work items per SM when (request, head) pairs are fewer than SMs
+                                   // (measured best of 1, 2, 3 on the long-context workload)
 constexpr int kMinChunk = 256;     // never split a sequence below this many tokens
 constexpr int kChunkAlign = 128;   // chunk starts are multiples of the KV tile
 
@@ -35,7 +42,7 @@ struct Layout {
   size_t plan_header = 0;     // PlanHeader
   size_t req_item_begin = 0;  // int32 [B]  first item of request r
   size_t req_chunks = 0;      // int32 [B]  chunks per KV head of request r
-  size_t pair_done = 0;       // int32 [B * Hkv] finished chunks per split (request, head)
+  size_t pair_done = 0;       // int32 [B * Hkv * 2] finished chunks per split (request, head, row group)
   size_t items = 0;           // WorkItem [max_items]
   size_t order = 0;           // int32 [max_items]  dispatch order of the items (largest first)
   size_t partials = 0;        // float [partial_cap]
@@ -51,6 +58,7 @@ struct PlanParams {
   int total_q_rows, total_draft;  // total_draft < 0: not checked (attention-only call)
   int with_attention;          // 0: offsets and validation only
   int target_items;
+  int max_rows_item;           // row groups of at most this many rows (rows per head <= 2 * this)
   int64_t max_items, partial_cap;
   const int32_t *draft_lens, *context_lens;
   const int64_t *request_ids;

@@ -173,11 +173,13 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo, ui
   return d;
 }
 
-// Instruction descriptor, kind::f16: fp32 accumulate, bf16 A and B, A K-major.
-__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool b_mn_major) {
+// Instruction descriptor, kind::f16: fp32 accumulate, bf16 A and B; an operand is K-major
+// unless its flag says MN-major (M, resp. N, the contiguous dimension in shared memory).
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool a_mn_major, bool b_mn_major) {
   return (1u << 4)                            // D format: f32
          | (1u << 7)                          // A format: bf16
          | (1u << 10)                         // B format: bf16
+         | ((a_mn_major ? 1u : 0u) << 15)     // A major-ness
          | ((b_mn_major ? 1u : 0u) << 16)     // B major-ness
          | ((uint32_t)(N >> 3) << 17)         // N / 8
          | ((uint32_t)(M >> 4) << 24);        // M / 16

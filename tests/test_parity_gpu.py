@@ -42,6 +42,9 @@ SMALL_CASES = [
     (3, "f32", 4, 4, 64, 1000, (0, 6), (0, 300)),
     (4, "bf16", 16, 16, 64, 777, (0, 5), (0, 200)),
     (5, "f32", 8, 2, 128, 3001, (0, 4), (0, 400)),
+    # 8 query heads per KV head and k up to 15: up to 128 rows per (request, head), cut into two
+    # row groups of at most 64 by the planner, with split chunks
+    (6, "bf16", 32, 4, 128, 2000, (8, 15), (0, 2500)),
 ]
 
 
