@@ -40,6 +40,7 @@
 #include "sm100_ptx.cuh"
 
 #include <cudaTypedefs.h>
+#include <mutex>
 #include <type_traits>
 
 namespace wisp {
@@ -924,13 +925,52 @@ cudaError_t attn_tc_setup() {
   return e;
 }
 
-cudaError_t attn_tc_launch(const AttnParams &p, int grid, cudaStream_t s) {
+namespace {
+
+// The four tensor maps of a (K pool, V pool, D, Hkv, num_blocks) are the same from step to step:
+// the last few sets are kept, so that a launch does not encode them again.
+struct PoolMaps {
+  const void *k = nullptr, *v = nullptr;
+  int D = 0, Hkv = 0, num_blocks = 0;
   alignas(64) CUtensorMap tk, tv, tk8, tv8;
-  cudaError_t e = encode_pool(&tk, p.k_cache, p.D, p.Hkv, p.num_blocks, 1);
-  if (e == cudaSuccess) e = encode_pool(&tv, p.v_cache, p.D, p.Hkv, p.num_blocks, 1);
-  if (e == cudaSuccess) e = encode_pool(&tk8, p.k_cache, p.D, p.Hkv, p.num_blocks, 8);
-  if (e == cudaSuccess) e = encode_pool(&tv8, p.v_cache, p.D, p.Hkv, p.num_blocks, 8);
+};
+constexpr int kMapCache = 8;
+PoolMaps g_maps[kMapCache];
+int g_maps_next = 0;
+std::mutex g_maps_mu;
+
+cudaError_t pool_maps(const AttnParams &p, PoolMaps *out) {
+  std::lock_guard<std::mutex> lk(g_maps_mu);
+  for (const PoolMaps &m : g_maps) {
+    if (m.k == p.k_cache && m.v == p.v_cache && m.D == p.D && m.Hkv == p.Hkv && m.num_blocks == p.num_blocks) {
+      *out = m;
+      return cudaSuccess;
+    }
+  }
+  PoolMaps m;
+  m.k = p.k_cache;
+  m.v = p.v_cache;
+  m.D = p.D;
+  m.Hkv = p.Hkv;
+  m.num_blocks = p.num_blocks;
+  cudaError_t e = encode_pool(&m.tk, p.k_cache, p.D, p.Hkv, p.num_blocks, 1);
+  if (e == cudaSuccess) e = encode_pool(&m.tv, p.v_cache, p.D, p.Hkv, p.num_blocks, 1);
+  if (e == cudaSuccess) e = encode_pool(&m.tk8, p.k_cache, p.D, p.Hkv, p.num_blocks, 8);
+  if (e == cudaSuccess) e = encode_pool(&m.tv8, p.v_cache, p.D, p.Hkv, p.num_blocks, 8);
   if (e != cudaSuccess) return e;
+  g_maps[g_maps_next] = m;
+  g_maps_next = (g_maps_next + 1) % kMapCache;
+  *out = m;
+  return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t attn_tc_launch(const AttnParams &p, int grid, cudaStream_t s) {
+  PoolMaps m;
+  const cudaError_t e = pool_maps(p, &m);
+  if (e != cudaSuccess) return e;
+  const CUtensorMap &tk = m.tk, &tv = m.tv, &tk8 = m.tk8, &tv8 = m.tv8;
   if (p.D == 128) {
     attn_tc_kernel<128><<<grid, kThreads, Cfg<128>::SMEM, s>>>(p, tk, tv, tk8, tv8);
   } else {
