@@ -102,14 +102,16 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
   if (!p.with_attention) return;
   __syncthreads();
 
-  // pass 2: chunk length so that sum over (r, h) of ceil(n_r / chunk_len) is about the item goal:
-  // one item per SM when there are at least as many (request, head) pairs as SMs (a longest-first
-  // order then balances whole sequences and few need the merge of split chunks), else
-  // kItemsPerSM items per SM
+  // pass 2: chunk length.  With at least as many (request, head) pairs as SMs, a longest-first
+  // order balances whole sequences: only a sequence longer than 5/4 of the average work per SM
+  // is cut (a split costs a merge of its chunks).  With fewer pairs than SMs, sequences are cut
+  // into about kItemsPerSM items per SM.
   const int64_t work = carry_n * p.Hkv;
   const int64_t sms = max(1, p.target_items / kItemsPerSM);
-  const int64_t goal = carry_v * p.Hkv >= sms ? sms : (int64_t)p.target_items;
+  const bool many_pairs = carry_v * p.Hkv >= sms;
+  const int64_t goal = many_pairs ? sms : (int64_t)p.target_items;
   int64_t chunk = (work + goal - 1) / goal;
+  if (many_pairs) chunk += chunk / 4;
   chunk = max64(chunk, kMinChunk);
   chunk = (chunk + kChunkAlign - 1) / kChunkAlign * kChunkAlign;
 
