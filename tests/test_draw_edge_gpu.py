@@ -1,0 +1,81 @@
+"""GPU: the extra-token draw (Eq. 3) when u * S lies next to an edge of the residual's CDF.
+
+The uniforms are placed about 1e-8 (relative) from an edge of the residual CDF: above the logging
+window of the parity tests, far below what fp32 weights or an fp32 normaliser could resolve.  The
+GPU's double-float weights and prefix sums must still give the fp64 oracle's token exactly.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2601_11652_gb300 import workload as wl
+from tests.gpu_util import SAMPLE_WINDOW
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.fail("GPU tests need a CUDA device")
+    from paper_2601_11652_gb300 import build
+    build.build()
+
+
+def _logit_row(batch, i):
+    row = batch.logits[i]
+    return row
+
+
+def _edge_uniforms(batch, ref, rng):
+    """For every request with a rejection, a float32 u next to an edge of its residual CDF."""
+    qs, ds = batch.q_row_start(), batch.draft_start()
+    out = {}
+    for r in range(batch.B):
+        L, k = int(ref["accepted_len"][r]), int(batch.draft_lens[r])
+        if L < 0 or L >= k:
+            continue
+        p = oracle.row_softmax(_logit_row(batch, qs[r] + L), batch.dtype)
+        q = batch.draft_probs[ds[r] + L].astype(np.float64)
+        res = np.maximum(p - q, 0.0)
+        tot = res.sum()
+        if not tot > 0:
+            continue
+        cdf = np.cumsum(res) / tot
+        # an edge in the middle of the mass, after an element of non-negligible weight
+        cand = np.nonzero((cdf > rng.uniform(0.2, 0.8)) & (res / tot > 1e-5))[0]
+        if len(cand) == 0:
+            continue
+        j = int(cand[0])
+        out[r] = np.float32(cdf[j])
+    return out
+
+
+@pytest.mark.parametrize("seed,V", [(11, 40000), (12, 6000)])
+def test_draw_next_to_a_cdf_edge_matches_the_oracle(seed, V):
+    from paper_2601_11652_gb300.device_batch import DeviceBatch
+    rng = np.random.default_rng(seed)
+    b = wl.make_small_batch(seed, B=8, Hq=8, Hkv=2, D=128, V=V, dtype="bf16", k_range=(3, 8), ctx_range=(0, 300))
+    ref = oracle.accept(b)
+    edges = _edge_uniforms(b, ref, rng)
+    assert len(edges) >= 3, "the seeds give requests with a rejection"
+    for r, u in edges.items():
+        b.sample_uniforms[r] = u
+    ref = oracle.accept(b)
+    # keep the edge requests whose margin is above the logging window (one float32 step off if not)
+    for r in list(edges):
+        if ref["sample_margin"][r] < SAMPLE_WINDOW:
+            b.sample_uniforms[r] = np.nextafter(b.sample_uniforms[r], np.float32(1.0))
+    ref = oracle.accept(b)
+    near = [r for r in edges if SAMPLE_WINDOW <= ref["sample_margin"][r] < 1e-6]
+    assert len(near) >= 3, [float(ref["sample_margin"][r]) for r in edges]
+    db = DeviceBatch.from_host(b)
+    db.step()
+    torch.cuda.synchronize()
+    code, rid = db.device_status()
+    assert code == 0, (code, rid)
+    got = db.results()
+    for r in near:
+        assert got["accepted_len"][r] == ref["accepted_len"][r]
+        assert got["next_token"][r] == ref["next_token"][r], (r, float(ref["sample_margin"][r]))
