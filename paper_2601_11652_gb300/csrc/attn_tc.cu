@@ -49,8 +49,10 @@ namespace {
 
 constexpr int kBT = 128;            // KV tokens per tile (the M of S^T)
 constexpr int kNR = kTcRowsPerItem; // query rows per item at most (64: the planner cuts larger sets)
-constexpr int kThreads = 384;       // warp 0 K producer, warp 1 MMA, warps 2-5 softmax, warp 6 item loader,
-                                    // warp 7 V producer, warps 8-11 epilogue
+constexpr int kThreads = 512;       // warp 0 K producer, warp 1 MMA, warps 2-5 softmax (rows 0-31), warp 6
+                                    // item loader, warp 7 V producer, warps 8-11 epilogue, warps 12-15
+                                    // softmax (rows 32-63)
+constexpr int kSoftmaxWarps = 8;
 constexpr uint32_t kTmemCols = 256; // S^T[2] at columns 0 / 64, O^T[2] at 128 / 192
 constexpr long long kWaitCycles = 4000000000LL;  // about two seconds: a wait that long is a failure
 constexpr float kTau = 8.0f;        // lazy rescale threshold (log2 units)
@@ -75,15 +77,14 @@ struct Cfg {
   static constexpr int OFF_P = OFF_V + NSV * KV_TILE;
   static constexpr int OFF_BAR = OFF_P + NP * P_BYTES;
   static constexpr int N_BAR = 2 * NSK + 2 * NSV + 8 + 2 * NP + 6 + 1 + 2 * RING + 5;
-  static constexpr int OFF_MW = (OFF_BAR + N_BAR * 8 + 15) / 16 * 16;  // float [4][64] per-warp row maxima
-  static constexpr int OFF_FW = OFF_MW + 4 * kNR * 4;                  // float [4][64] per-warp rescale factors
-  static constexpr int OFF_RED = OFF_FW + 4 * kNR * 4;                 // float [4][64] tile maxima per warp
-  static constexpr int OFF_FLAG = OFF_RED + 4 * kNR * 4;               // uint32 [2][4] exceed flags per warp
-  static constexpr int OFF_HL = OFF_FLAG + 32;                         // float [2][4][64] row-sum shares per warp
+  static constexpr int OFF_MW = (OFF_BAR + N_BAR * 8 + 15) / 16 * 16;  // float [8][32] per-warp row maxima
+  static constexpr int OFF_FW = OFF_MW + kSoftmaxWarps * 32 * 4;       // float [8][32] per-warp rescale factors
+  static constexpr int OFF_RED = OFF_FW + kSoftmaxWarps * 32 * 4;      // float [4][64] tile maxima per quadrant
+  static constexpr int OFF_FLAG = OFF_RED + 4 * kNR * 4;               // uint32 [2][8] exceed votes per warp
+  static constexpr int OFF_HL = OFF_FLAG + 64;                         // float [2][4][64] row-sum shares per quadrant
   static constexpr int OFF_HM = OFF_HL + 2 * 4 * kNR * 4;              // float [2][64] row reference maxima
   static constexpr int OFF_EM = OFF_HM + 2 * kNR * 4;                  // float [2][64] merge: max, 1 / sum
-  static constexpr int OFF_TR = OFF_EM + 2 * kNR * 4;                  // float [4][32][33] per-warp transposes
-  static constexpr int OFF_MISC = OFF_TR + 4 * 32 * 33 * 4;            // tmem base, flags
+  static constexpr int OFF_MISC = OFF_EM + 2 * kNR * 4;                // tmem base, flags
   static constexpr int OFF_RING = OFF_MISC + 64;                       // RING x (index, WorkItem)
   static constexpr int SMEM = OFF_RING + RING * 64 + 1024;             // + slack to align the base to 1024
   static_assert(SMEM <= 227 * 1024, "shared memory of one CTA on sm_103a");
@@ -118,18 +119,22 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   return *reinterpret_cast<uint32_t *>(&v);
 }
 
-// Reductions over the 32 lanes of a warp through a padded shared 32 x 33 scratch: on return lane i
-// holds the sum (max) over all lanes of v[i].  Conflict-free both ways.
+// Transposing reductions over the 32 lanes of a warp (v is consumed): on return lane i holds the
+// sum (max) over all lanes of v[i].  31 shuffles for 32 values.
 template <bool MAX>
-__device__ __forceinline__ float warp_transpose_reduce(const float (&v)[32], float *tr, int lane) {
+__device__ __forceinline__ float warp_transpose_reduce(float (&v)[32], int lane) {
 #pragma unroll
-  for (int i = 0; i < 32; ++i) tr[lane * 33 + i] = v[i];
-  __syncwarp();
-  float r = MAX ? -INFINITY : 0.0f;
+  for (int w = 16; w >= 1; w >>= 1) {
+    const bool up = (lane & w) != 0;
 #pragma unroll
-  for (int i = 0; i < 32; ++i) r = MAX ? fmaxf(r, tr[i * 33 + lane]) : r + tr[i * 33 + lane];
-  __syncwarp();
-  return r;
+    for (int i = 0; i < w; ++i) {
+      const float keep = up ? v[i + w] : v[i];
+      const float send = up ? v[i] : v[i + w];
+      const float got = __shfl_xor_sync(0xffffffffu, send, w);
+      v[i] = MAX ? fmaxf(keep, got) : keep + got;
+    }
+  }
+  return v[0];
 }
 
 }  // namespace
@@ -162,8 +167,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   B.it_full = B.mma_done + 1;
   B.it_empty = B.it_full + C::RING;
   B.egrp = B.it_empty + C::RING;
-  B.sm_sync = B.egrp + 1;       // the four softmax warps, once per tile
-  B.sm_sync2 = B.sm_sync + 1;   // the four softmax warps, once per tile that moves a reference max
+  B.sm_sync = B.egrp + 1;       // the softmax warps, once per tile
+  B.sm_sync2 = B.sm_sync + 1;   // the softmax warps, once per tile that moves a reference max
   B.fin = B.sm_sync2 + 1;       // every warp, once: its last access to TMEM is done
   B.claim = B.fin + 1;          // the K producer, once per item, a few tiles before the item's end
   static_assert(2 * C::NSK + 2 * C::NSV + 8 + 2 * C::NP + 6 + 1 + 2 * C::RING + 5 <= C::N_BAR, "barrier count");
@@ -174,7 +179,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   float *s_em = reinterpret_cast<float *>(smem + C::OFF_EM);
   float *s_hl = reinterpret_cast<float *>(smem + C::OFF_HL);
   float *s_hm = reinterpret_cast<float *>(smem + C::OFF_HM);
-  float *s_tr = reinterpret_cast<float *>(smem + C::OFF_TR);
   uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + C::OFF_MISC);
   volatile int *s_abort = reinterpret_cast<volatile int *>(smem + C::OFF_MISC + 4);
   volatile int *s_last = reinterpret_cast<volatile int *>(smem + C::OFF_MISC + 8);
@@ -200,25 +204,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::mbar_init(B.q_full + b, 1);
       ptx::mbar_init(B.q_empty + b, 1);
       ptx::mbar_init(B.s_full + b, 1);
-      ptx::mbar_init(B.s_empty + b, 4);
+      ptx::mbar_init(B.s_empty + b, kSoftmaxWarps);
     }
     for (int b = 0; b < C::NP; ++b) {
-      ptx::mbar_init(B.p_full + b, 4);
+      ptx::mbar_init(B.p_full + b, kSoftmaxWarps);
       ptx::mbar_init(B.o_full + b, 1);
     }
     for (int b = 0; b < 2; ++b) {
       ptx::mbar_init(B.o_empty + b, 4);  // the four epilogue warps
       ptx::mbar_init(B.o_done + b, 1);
-      ptx::mbar_init(B.ep_full + b, 4);  // the four softmax warps
+      ptx::mbar_init(B.ep_full + b, kSoftmaxWarps);
     }
     ptx::mbar_init(B.mma_done, 1);
     for (int i = 0; i < C::RING; ++i) {
       ptx::mbar_init(B.it_full + i, 1);
-      ptx::mbar_init(B.it_empty + i, 11);  // KV producers, MMA thread, softmax and epilogue warps
+      ptx::mbar_init(B.it_empty + i, 3 + kSoftmaxWarps + 4);  // KV producers, MMA, softmax and epilogue warps
     }
     ptx::mbar_init(B.egrp, 4);      // the four epilogue warps
-    ptx::mbar_init(B.sm_sync, 4);   // the four softmax warps
-    ptx::mbar_init(B.sm_sync2, 4);
+    ptx::mbar_init(B.sm_sync, kSoftmaxWarps);
+    ptx::mbar_init(B.sm_sync2, kSoftmaxWarps);
     ptx::mbar_init(B.fin, kThreads / 32);
     ptx::mbar_init(B.claim, 1);
     *s_abort = 0;
@@ -499,7 +503,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       while (!ptx::mbar_try_wait(B.mma_done, 0) && clock64() - t0 < kWaitCycles) {
       }
     }
-  } else if (warp >= 8) {
+  } else if (warp >= 8 && warp < 12) {
     // ------------------------------------------------------------------ epilogue warps
     // One warp per TMEM lane quadrant: thread d (lane d of O^T) owns head-dim index d of every row.
     // Item li's O^T (buffer li & 1) is read once the softmax warps have handed the item over and
@@ -640,14 +644,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!ok && lane == 0) report(p.status, WISP_DEV_TIMEOUT, p.request_ids, 0);
   } else {
     // ------------------------------------------------------------------ softmax warps
-    const int qd = warp & 3;          // TMEM lane quadrant of this warp: keys 32*qd .. 32*qd + 31 of a tile
+    // Two groups of four: warps 2-5 take rows 0-31 of every item, warps 12-15 rows 32-63 (and only
+    // keep in step for items of at most 32 rows).  Within a group, one warp per TMEM lane quadrant,
+    // i.e. 32 keys of each tile: a thread holds one key's scores for the group's 32 rows.
+    const int qd = warp & 3;                  // TMEM lane quadrant: keys 32*qd .. 32*qd + 31 of a tile
+    const int grp = warp >= 12 ? 1 : 0;       // row chunk: rows 32*grp .. 32*grp + 31
+    const int sw8 = grp * 4 + qd;             // index of this warp among the eight
     const uint32_t lane_addr = (uint32_t)(qd * 32) << 16;
     const float scale_log2 = 1.4426950408889634f / sqrtf((float)D);
-    float *mw = s_mw + qd * kNR;      // this warp's copy of the rows' reference maxima
-    float *fw = s_fw + qd * kNR;      // this warp's copy of the rescale factors
-    float *tr = s_tr + qd * 32 * 33;  // this warp's transpose scratch
-    uint32_t n = 0, nf = 0;           // tiles so far; tiles that moved a reference max
-    int li = 0;                       // items so far: item li accumulates into O buffer li & 1
+    float *mw = s_mw + sw8 * 32;              // this warp's copy of its rows' reference maxima
+    float *fw = s_fw + sw8 * 32;              // this warp's copy of its rows' rescale factors
+    const int r0 = 32 * grp;                  // first row of the chunk
+    uint32_t n = 0, nf = 0;                   // tiles so far; tiles that moved a reference max
+    int li = 0;                               // items so far: item li accumulates into O buffer li & 1
     bool ok = true;
     for (uint32_t j = 0; ok; ++j) {
       const int slot = j % C::RING;
@@ -660,137 +669,122 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int ob = li & 1;
       const uint32_t o_col = 128 + ob * kNR;
       const int ntiles = (w.t1 - w.t0 + kBT - 1) / kBT;
-      const int nu = (w.rows + 15) / 16 * 2;  // 8-row units the MMA reads (its N / 8)
+      // 8-row units of this chunk that the MMA reads (its N / 8 minus the chunk's offset)
+      const int nu = min(4, max(0, (w.rows + 15) / 16 * 2 - 4 * grp));
+      const bool active = nu > 0;
+      const int jmax = w.rows - r0;          // rows of the item in this chunk (may be <= 0)
       mw[lane] = -INFINITY;
-      mw[lane + 32] = -INFINITY;
       __syncwarp();
-
-      // the tile loop, specialised for the 32-row chunks of the item
-      auto run_tiles = [&](auto nc_tag) -> bool {
-        constexpr int NC = decltype(nc_tag)::value;
-        float lp[NC][32];  // this thread's (key's) share of every row sum
+      float lp[32];  // this thread's (key's) share of every row sum of the chunk
 #pragma unroll
-        for (int c = 0; c < NC; ++c)
-#pragma unroll
-          for (int i = 0; i < 32; ++i) lp[c][i] = 0.0f;
-        for (int t = 0; t < ntiles; ++t, ++n) {
-          const int sb = n & 1;
-          if (!wait_bar(B.s_full + sb, (n >> 1) & 1, s_abort)) return false;
-          ptx::tc_fence_after();
-          // P buffer n % NP is free again once PV(n - NP) is done (this thread waited PV(n - 2NP)
-          // before, and PV(n) needs the P(n) it is about to publish: the parity is exact)
-          const int pbuf = (int)(n % C::NP);
-          if (n >= (uint32_t)C::NP && !wait_bar(B.o_full + pbuf, ((n - C::NP) / C::NP) & 1, s_abort)) return false;
-          // this key's row of P^T: 128 bytes (64 rows, bf16), 16-byte units swizzled by key & 7
-          uint8_t *prow = smem + C::OFF_P + pbuf * C::P_BYTES + (qd * 32 + lane) * 128;
-          const int sw = lane & 7;
-          // causal mask: key tok is visible to row jr iff tok <= ctx + (row0 + jr) / g, i.e.
-          // row0 + jr >= g * (tok - ctx); keys past the item and rows past `rows` are masked too
-          const int tok = w.t0 + t * kBT + qd * 32 + lane;
-          const int jmin = tok >= w.t1 ? kNR : max(0, g * (tok - w.ctx) - w.row0);
-          const int jmax = w.rows;
+      for (int i = 0; i < 32; ++i) lp[i] = 0.0f;
+      for (int t = 0; t < ntiles && ok; ++t, ++n) {
+        const int sb = n & 1;
+        if (!wait_bar(B.s_full + sb, (n >> 1) & 1, s_abort)) { ok = false; break; }
+        ptx::tc_fence_after();
+        const int pbuf = (int)(n % C::NP);
+        uint8_t *prow = smem + C::OFF_P + pbuf * C::P_BYTES + (qd * 32 + lane) * 128;
+        const int sw = lane & 7;
+        // causal mask: key tok is visible to row jr iff tok <= ctx + (row0 + jr) / g, i.e.
+        // row0 + jr >= g * (tok - ctx); keys past the item and rows past `rows` are masked too
+        const int tok = w.t0 + t * kBT + qd * 32 + lane;
+        const int jmin = (tok >= w.t1 ? kNR : max(0, g * (tok - w.ctx) - w.row0)) - r0;
+        float emax = 0.0f;
+        if (active) {
+          // P buffer n % NP is free again once PV(n - NP) is done: the other group's wait or this
+          // warp's own one covered PV(n - 2NP), and PV(n) needs the P(n) about to be published,
+          // so the parity is exact
+          if (n >= (uint32_t)C::NP && !wait_bar(B.o_full + pbuf, ((n - C::NP) / C::NP) & 1, s_abort)) {
+            ok = false;
+            break;
+          }
           // P = 2^(s - m) against the current reference maxima (masked: 0), written straight to the
           // P buffer and added to the row-sum shares; the vote asks whether any P exceeds 2^kTau
           // (then the tile is redone below with new references)
-          float emax = 0.0f;
+          uint32_t x[32];
+          ptx::tmem_ld32(tmem + lane_addr + sb * kNR + r0, x);
+          ptx::tmem_wait_ld();
 #pragma unroll
-          for (int c = 0; c < NC; ++c) {
-            uint32_t x[32];
-            ptx::tmem_ld32(tmem + lane_addr + sb * kNR + 32 * c, x);
-            ptx::tmem_wait_ld();
+          for (int u = 0; u < 4; ++u) {
+            if (u < nu) {
+              uint32_t pk[4];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              if (4 * c + u < nu) {
-                uint32_t pk[4];
+              for (int h = 0; h < 2; ++h) {
+                const int i0 = 8 * u + 4 * h;
+                const float4 m4 = reinterpret_cast<const float4 *>(mw + i0)[0];
+                const float mm[4] = {m4.x, m4.y, m4.z, m4.w};
+                float e[4];
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                  const int i0 = 8 * u + 4 * h;
-                  const float4 m4 = reinterpret_cast<const float4 *>(mw + 32 * c + i0)[0];
-                  const float mm[4] = {m4.x, m4.y, m4.z, m4.w};
-                  float e[4];
-#pragma unroll
-                  for (int q = 0; q < 4; ++q) {
-                    const int jr = 32 * c + i0 + q;
-                    const float v = ptx::ex2(fmaf(__uint_as_float(x[i0 + q]), scale_log2, -mm[q]));
-                    e[q] = (jr >= jmin && jr < jmax) ? v : 0.0f;
-                    emax = fmaxf(emax, e[q]);
-                    lp[c][i0 + q] += e[q];
-                  }
-                  pk[2 * h] = pack_bf16(e[0], e[1]);
-                  pk[2 * h + 1] = pack_bf16(e[2], e[3]);
+                for (int q = 0; q < 4; ++q) {
+                  const int jr = i0 + q;
+                  const float v = ptx::ex2(fmaf(__uint_as_float(x[i0 + q]), scale_log2, -mm[q]));
+                  e[q] = (jr >= jmin && jr < jmax) ? v : 0.0f;
+                  emax = fmaxf(emax, e[q]);
+                  lp[i0 + q] += e[q];
                 }
-                *reinterpret_cast<uint4 *>(prow + (((4 * c + u) ^ sw) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                pk[2 * h] = pack_bf16(e[0], e[1]);
+                pk[2 * h + 1] = pack_bf16(e[2], e[3]);
               }
+              *reinterpret_cast<uint4 *>(prow + (((4 * grp + u) ^ sw) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
             }
           }
-          // the four warps' votes, double-buffered by tile parity (NaN never wins fmaxf, and a
-          // visible key of a row without a reference yet gives +inf)
-          const uint32_t vote = __ballot_sync(0xffffffffu, !(emax <= kExpTau));
-          if (lane == 0) {
-            s_flag[(n & 1) * 4 + qd] = vote;
-            ptx::mbar_arrive(B.sm_sync);
-          }
-          if (!wait_bar(B.sm_sync, n & 1, s_abort)) return false;
-          const bool any = (s_flag[(n & 1) * 4] | s_flag[(n & 1) * 4 + 1] | s_flag[(n & 1) * 4 + 2] |
-                            s_flag[(n & 1) * 4 + 3]) != 0;
-          if (any) {
-            // new references: exact tile maxima per row (over this warp's 32 keys through the
-            // transpose scratch, then over the four warps), from the scores read again
+        }
+        // the eight warps' votes, double-buffered by tile parity (NaN never wins fmaxf, and a
+        // visible key of a row without a reference yet gives +inf)
+        const uint32_t vote = __ballot_sync(0xffffffffu, !(emax <= kExpTau));
+        if (lane == 0) {
+          s_flag[(n & 1) * 8 + sw8] = vote;
+          ptx::mbar_arrive(B.sm_sync);
+        }
+        if (!wait_bar(B.sm_sync, n & 1, s_abort)) { ok = false; break; }
+        uint32_t anyv = 0;
 #pragma unroll
-            for (int c = 0; c < NC; ++c) {
+        for (int k8 = 0; k8 < 8; ++k8) anyv |= s_flag[(n & 1) * 8 + k8];
+        if (anyv != 0) {
+          // new references: exact tile maxima per row (over this warp's 32 keys, then over the
+          // group's four quadrants), from the scores read again
+          if (active) {
+            uint32_t x[32];
+            ptx::tmem_ld32(tmem + lane_addr + sb * kNR + r0, x);
+            ptx::tmem_wait_ld();
+            float sv[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              sv[i] = (i >= jmin && i < jmax) ? __uint_as_float(x[i]) * scale_log2 : -INFINITY;  // scale > 0
+            s_red[qd * kNR + r0 + lane] = warp_transpose_reduce<true>(sv, lane);
+          }
+          __syncwarp();
+          if (lane == 0) ptx::mbar_arrive(B.sm_sync2);
+          if (!wait_bar(B.sm_sync2, nf & 1, s_abort)) { ok = false; break; }
+          ++nf;
+          if (active) {
+            // this tile's P leaves the shares (a row without a reference had nothing yet)
+            {
               uint32_t x[32];
-              ptx::tmem_ld32(tmem + lane_addr + sb * kNR + 32 * c, x);
+              ptx::tmem_ld32(tmem + lane_addr + sb * kNR + r0, x);
               ptx::tmem_wait_ld();
 #pragma unroll
               for (int i = 0; i < 32; ++i) {
-                const int jr = 32 * c + i;
-                tr[lane * 33 + i] = (jr >= jmin && jr < jmax) ? __uint_as_float(x[i]) * scale_log2 : -INFINITY;  // scale > 0
-              }
-              __syncwarp();
-              float tm = -INFINITY;
-#pragma unroll
-              for (int i = 0; i < 32; ++i) tm = fmaxf(tm, tr[i * 33 + lane]);
-              s_red[qd * kNR + 32 * c + lane] = tm;
-              __syncwarp();
-            }
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(B.sm_sync2);
-            if (!wait_bar(B.sm_sync2, nf & 1, s_abort)) return false;
-            ++nf;
-            // take this tile's P back out of the shares (a row without a reference had nothing yet)
-#pragma unroll
-            for (int c = 0; c < NC; ++c) {
-              uint32_t x[32];
-              ptx::tmem_ld32(tmem + lane_addr + sb * kNR + 32 * c, x);
-              ptx::tmem_wait_ld();
-#pragma unroll
-              for (int i = 0; i < 32; ++i) {
-                const int jr = 32 * c + i;
-                const float mo = mw[jr];
+                const float mo = mw[i];
                 const float v = ptx::ex2(fmaf(__uint_as_float(x[i]), scale_log2, -mo));
-                const float eo = (jr >= jmin && jr < jmax) ? v : 0.0f;
-                lp[c][i] = mo == -INFINITY ? 0.0f : lp[c][i] - eo;
+                const float eo = (i >= jmin && i < jmax) ? v : 0.0f;
+                lp[i] = mo == -INFINITY ? 0.0f : lp[i] - eo;
               }
             }
             __syncwarp();
-            // every warp derives the same new maxima and factors from the same values
-            bool moved = false;
-#pragma unroll
-            for (int c = 0; c < NC; ++c) {
-              const int jl = 32 * c + lane;
-              const float tmax = fmaxf(fmaxf(s_red[jl], s_red[kNR + jl]), fmaxf(s_red[2 * kNR + jl], s_red[3 * kNR + jl]));
-              const float mo = mw[jl];
-              const float mn = tmax > mo + kTau ? tmax : mo;
-              fw[jl] = mn == mo ? 1.0f : (mo == -INFINITY ? 0.0f : ptx::ex2(mo - mn));
-              moved |= mn != mo && mo != -INFINITY;
-              mw[jl] = mn;
-            }
+            // every warp of the group derives the same new maxima and factors from the same values
+            const int jl = r0 + lane;
+            const float tmax = fmaxf(fmaxf(s_red[jl], s_red[kNR + jl]), fmaxf(s_red[2 * kNR + jl], s_red[3 * kNR + jl]));
+            const float mo = mw[lane];
+            const float mn = tmax > mo + kTau ? tmax : mo;
+            fw[lane] = mn == mo ? 1.0f : (mo == -INFINITY ? 0.0f : ptx::ex2(mo - mn));
+            const bool moved = mn != mo && mo != -INFINITY;
+            mw[lane] = mn;
             __syncwarp();
             // P again against the new references: shares rescaled, P rewritten
-#pragma unroll
-            for (int c = 0; c < NC; ++c) {
+            {
               uint32_t x[32];
-              ptx::tmem_ld32(tmem + lane_addr + sb * kNR + 32 * c, x);
+              ptx::tmem_ld32(tmem + lane_addr + sb * kNR + r0, x);
               ptx::tmem_wait_ld();
 #pragma unroll
               for (int u = 0; u < 4; ++u) {
@@ -800,67 +794,58 @@ __global__ void __launch_bounds__(kThreads, 1)
                   float e[4];
 #pragma unroll
                   for (int q = 0; q < 4; ++q) {
-                    const int i = 8 * u + 4 * h + q, jr = 32 * c + i;
-                    const float v = ptx::ex2(fmaf(__uint_as_float(x[i]), scale_log2, -mw[jr]));
-                    e[q] = (jr >= jmin && jr < jmax) ? v : 0.0f;
-                    lp[c][i] = fmaf(lp[c][i], fw[jr], e[q]);
+                    const int i = 8 * u + 4 * h + q;
+                    const float v = ptx::ex2(fmaf(__uint_as_float(x[i]), scale_log2, -mw[i]));
+                    e[q] = (i >= jmin && i < jmax) ? v : 0.0f;
+                    lp[i] = fmaf(lp[i], fw[i], e[q]);
                   }
                   pk[2 * h] = pack_bf16(e[0], e[1]);
                   pk[2 * h + 1] = pack_bf16(e[2], e[3]);
                 }
-                if (4 * c + u < nu)
-                  *reinterpret_cast<uint4 *>(prow + (((4 * c + u) ^ sw) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                if (u < nu)
+                  *reinterpret_cast<uint4 *>(prow + (((4 * grp + u) ^ sw) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
               }
             }
-            // O^T, if it holds earlier tiles of the item, moves to the new references; the rescale
-            // needs PV(n-1) complete and precedes PV(n)
+            // this chunk's O^T columns, if they hold earlier tiles of the item, move to the new
+            // references; the rescale needs PV(n-1) complete and precedes PV(n)
             if (t > 0 && __any_sync(0xffffffffu, moved)) {
-              // PV(m) completes barrier o_full[m % NP] for the (m / NP)-th time; this thread has
-              // waited PV(n-NP) already and PV(n-1+NP) needs P(n-1+NP), so the parity names PV(n-1)
-              if (!wait_bar(B.o_full + (n - 1) % C::NP, ((n - 1) / C::NP) & 1, s_abort)) return false;
+              // PV(m) completes barrier o_full[m % NP] for the (m / NP)-th time; PV(n-1-NP) was
+              // waited for (by this warp or, through the tile votes, by the other group) and
+              // PV(n-1+NP) needs P(n-1+NP), so the parity names PV(n-1)
+              if (!wait_bar(B.o_full + (n - 1) % C::NP, ((n - 1) / C::NP) & 1, s_abort)) { ok = false; break; }
               ptx::tc_fence_after();
 #pragma unroll
-              for (int c = 0; c < 2 * NC; ++c) {
+              for (int c = 0; c < 2; ++c) {
                 uint32_t y[16];
-                ptx::tmem_ld16(tmem + lane_addr + o_col + 16 * c, y);
+                ptx::tmem_ld16(tmem + lane_addr + o_col + r0 + 16 * c, y);
                 ptx::tmem_wait_ld();
 #pragma unroll
                 for (int i = 0; i < 16; ++i) y[i] = __float_as_uint(__uint_as_float(y[i]) * fw[16 * c + i]);
-                ptx::tmem_st16(tmem + lane_addr + o_col + 16 * c, y);
+                ptx::tmem_st16(tmem + lane_addr + o_col + r0 + 16 * c, y);
               }
               ptx::tmem_wait_st();
             }
           }
-          // S^T(n) has been read: its TMEM buffer may be overwritten by S^T(n+2); P(n) is published
-          ptx::tc_fence_before();
-          ptx::fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            ptx::mbar_arrive(B.s_empty + sb);
-            ptx::mbar_arrive(B.p_full + pbuf);
-          }
         }
-        // ---- hand the item over to the epilogue warps: this warp's share of each row sum and the
-        // reference maxima.  The epilogue of item li - 2 (same buffers) must be done with them.
-        float lsh[NC];
-#pragma unroll
-        for (int c = 0; c < NC; ++c) lsh[c] = warp_transpose_reduce<false>(lp[c], tr, lane);
-        if (!wait_bar(B.o_empty + ob, ((li >> 1) & 1) ^ 1, s_abort)) return false;
-#pragma unroll
-        for (int c = 0; c < NC; ++c) {
-          s_hl[(ob * 4 + qd) * kNR + 32 * c + lane] = lsh[c];
-          if (qd == 0) s_hm[ob * kNR + 32 * c + lane] = mw[32 * c + lane];
-        }
+        // S^T(n) has been read: its TMEM buffer may be overwritten by S^T(n+2); P(n) is published
+        ptx::tc_fence_before();
+        ptx::fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0) ptx::mbar_arrive(B.ep_full + ob);
-        return true;
-      };
-      if (w.rows <= 32) {
-        ok = run_tiles(std::integral_constant<int, 1>{});
-      } else {
-        ok = run_tiles(std::integral_constant<int, 2>{});
+        if (lane == 0) {
+          ptx::mbar_arrive(B.s_empty + sb);
+          ptx::mbar_arrive(B.p_full + pbuf);
+        }
       }
       if (!ok) break;
+      // ---- hand the item over to the epilogue warps: this quadrant's share of each row sum of
+      // the chunk, and the reference maxima.  The epilogue of item li - 2 (same buffers) must be
+      // done with them.
+      const float lsh = warp_transpose_reduce<false>(lp, lane);
+      if (!wait_bar(B.o_empty + ob, ((li >> 1) & 1) ^ 1, s_abort)) { ok = false; break; }
+      s_hl[(ob * 4 + qd) * kNR + r0 + lane] = lsh;
+      if (qd == 0) s_hm[ob * kNR + r0 + lane] = mw[lane];
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(B.ep_full + ob);
       ++li;
     }
     if (!ok && lane == 0) report(p.status, WISP_DEV_TIMEOUT, p.request_ids, 0);
