@@ -195,7 +195,7 @@ PlanParams plan_params(const wisp_attn_args *a, const wisp_accept_args *c, void 
   return pp;
 }
 
-wisp_status launch_attention(const wisp_attn_args *a, void *ws, const Layout &L, cudaStream_t s) {
+wisp_status launch_attention(const wisp_attn_args *a, void *ws, const Layout &L, cudaStream_t s, bool pdl) {
   AttnParams ap;
   ap.B = a->B;
   ap.Hq = a->Hq;
@@ -225,7 +225,7 @@ wisp_status launch_attention(const wisp_attn_args *a, void *ws, const Layout &L,
     const int grid = (int)(L.max_items < L.target_items / kItemsPerSM ? L.max_items : L.target_items / kItemsPerSM);
     // the work counter lives in the plan header written by the planner on this stream
     // split items are merged inside the kernel by the last chunk to finish
-    return attn_tc_launch(ap, grid, s) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
+    return attn_tc_launch(ap, grid, s, pdl) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
   }
   if (attn_simt_launch(ap, bf, (int)L.max_items, s) != cudaSuccess) return WISP_ERR_CUDA;
   return attn_combine_launch(ap, bf, s) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
@@ -337,7 +337,8 @@ wisp_status wisp_verify_attention(const wisp_attn_args *attn, void *ws, size_t w
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if ((st = launch_plan(attn, nullptr, ws, L, s)) != WISP_OK) return st;
   if (attn->B == 0) return WISP_OK;
-  return launch_attention(attn, ws, L, s);
+  // alone on the stream after the planner: the attention CTAs set up while the planner runs
+  return launch_attention(attn, ws, L, s, true);
 }
 
 wisp_status wisp_verify_accept(const wisp_accept_args *acc, void *ws, size_t ws_bytes, void *stream) {
@@ -392,7 +393,8 @@ wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args 
   // join what was forked even after a failed launch, so that `s` never runs ahead of `side`
   const bool joined = cudaEventRecord(d.ev_join, d.side) == cudaSuccess;
   ok = ok && launch_plan(attn, acc, ws, L, s) == WISP_OK;
-  ok = ok && launch_attention(attn, ws, L, s) == WISP_OK;
+  // no programmatic launch here: the row statistics should have the SMs while the planner runs
+  ok = ok && launch_attention(attn, ws, L, s, false) == WISP_OK;
   const bool waited = joined && cudaStreamWaitEvent(s, d.ev_join, 0) == cudaSuccess;
   ok = ok && waited && accept_walk_launch(ap, bf, s) == cudaSuccess;
   return ok && waited ? WISP_OK : WISP_ERR_CUDA;

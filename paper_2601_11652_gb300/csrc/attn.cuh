@@ -27,6 +27,9 @@ cudaError_t attn_simt_launch(const AttnParams &p, bool bf16, int grid, cudaStrea
 cudaError_t attn_combine_launch(const AttnParams &p, bool bf16, cudaStream_t s);
 // tcgen05 / TMA kernel for bf16 KV, D in {64, 128}; `grid` persistent CTAs
 cudaError_t attn_tc_setup();
-cudaError_t attn_tc_launch(const AttnParams &p, int grid, cudaStream_t s);
+// pdl: programmatic dependent launch (the CTAs' set-up overlaps the previous kernel on `s`, which
+// the kernel waits for before it reads the plan); off where another stream's kernel should get the
+// SMs first
+cudaError_t attn_tc_launch(const AttnParams &p, int grid, cudaStream_t s, bool pdl);
 
 }  // namespace wisp

@@ -40,6 +40,7 @@
 #include "sm100_ptx.cuh"
 
 #include <cudaTypedefs.h>
+#include <cstring>
 #include <mutex>
 #include <type_traits>
 
@@ -244,6 +245,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   ptx::tc_fence_after();
   const uint32_t tmem = *s_tmem;
 
+  // everything above may overlap the planner (programmatic dependent launch); the plan is read
+  // only once the planner's grid has completed and its writes are visible
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int n_items = p.header->n_items;
   const int g = p.Hq / p.Hkv;
 
@@ -951,17 +955,29 @@ cudaError_t pool_maps(const AttnParams &p, PoolMaps *out) {
 
 }  // namespace
 
-cudaError_t attn_tc_launch(const AttnParams &p, int grid, cudaStream_t s) {
+cudaError_t attn_tc_launch(const AttnParams &p, int grid, cudaStream_t s, bool pdl) {
   PoolMaps m;
   const cudaError_t e = pool_maps(p, &m);
   if (e != cudaSuccess) return e;
   const CUtensorMap &tk = m.tk, &tv = m.tv, &tk8 = m.tk8, &tv8 = m.tv8;
+  // programmatic dependent launch: the CTAs' set-up overlaps the kernel before this one (the
+  // planner), which the kernel waits for before it reads the plan
+  cudaLaunchConfig_t cfg;
+  std::memset(&cfg, 0, sizeof cfg);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
   if (p.D == 128) {
-    attn_tc_kernel<128><<<grid, kThreads, Cfg<128>::SMEM, s>>>(p, tk, tv, tk8, tv8);
-  } else {
-    attn_tc_kernel<64><<<grid, kThreads, Cfg<64>::SMEM, s>>>(p, tk, tv, tk8, tv8);
+    cfg.dynamicSmemBytes = Cfg<128>::SMEM;
+    return cudaLaunchKernelEx(&cfg, attn_tc_kernel<128>, p, tk, tv, tk8, tv8);
   }
-  return cudaGetLastError();
+  cfg.dynamicSmemBytes = Cfg<64>::SMEM;
+  return cudaLaunchKernelEx(&cfg, attn_tc_kernel<64>, p, tk, tv, tk8, tv8);
 }
 
 }  // namespace wisp

@@ -47,6 +47,9 @@ __device__ int64_t block_scan(int64_t v, int64_t *s_warp, int64_t *total) {
 }  // namespace
 
 __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
+  // a kernel launched after this one with programmatic stream serialization (the attention) may
+  // start its own set-up now; it reads the plan only after waiting for this grid to complete
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   __shared__ int64_t s_warp[32];
   const int tid = threadIdx.x;
   const int g = p.Hq > 0 && p.Hkv > 0 ? p.Hq / p.Hkv : 1;
