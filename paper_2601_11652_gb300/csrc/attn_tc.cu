@@ -12,8 +12,9 @@
 //
 // Persistent CTAs (one per SM) take work items (request, KV head, key chunk, row group) from a
 // global counter, in the planner's longest-first order.  Warp roles in a CTA:
-//   * warp 6 (item loader) takes the next item, publishes it to the other warps through a 4-slot
-//     shared ring, and copies its query rows into one of two shared Q buffers (128-byte-swizzled,
+//   * warp 6 (item loader) takes the next item just in time (when the K producer is three tiles
+//     from the end of the current one), publishes it to the other warps through a 4-slot shared
+//     ring, and copies its query rows into one of two shared Q buffers (128-byte-swizzled,
 //     K-major: the B operand of S^T);
 //   * warps 0 and 7 (K and V producers) stream the item's K and V tiles of 128 tokens with TMA
 //     tiled loads into two rings: one 16 KB box per 64-wide half of the head dim when the tile's
@@ -23,19 +24,21 @@
 //   * warp 1 (one thread) issues tcgen05.mma: S^T into one of two TMEM tiles (key t in TMEM lane
 //     t, query row j in column j), and O^T into the item's TMEM accumulator (head-dim index d in
 //     lane d, row j in column j; two accumulators alternating between items);
-//   * warps 2-5 (softmax), one per TMEM lane quadrant, i.e. 32 keys of each tile per warp: a thread
-//     holds one key's scores for all rows.  The rows' reference maxima live in shared memory; a
-//     tile whose scores exceed a reference by more than 2^8 anywhere (the first tile of an item
-//     always does) makes the four warps agree on new maxima (exact per-row tile maxima) and, if O
-//     holds earlier tiles, rescale the O^T columns in TMEM.  Each thread writes its key's P row
-//     (bf16, MN-major, swizzled: the B operand of the PV product) and keeps its share of every
-//     row sum;
+//   * warps 2-5 and 12-15 (softmax): the first group takes rows 0-31 of an item, the second rows
+//     32-63; within a group one warp per TMEM lane quadrant, i.e. 32 keys of each tile per warp: a
+//     thread holds one key's scores for the group's rows.  The rows' reference maxima live in
+//     shared memory; a tile whose scores exceed a reference by more than 2^8 anywhere (the first
+//     tile of an item always does) makes the warps agree on new maxima (exact per-row tile
+//     maxima) and, if O holds earlier tiles, rescale their O^T columns in TMEM.  Each thread
+//     writes its key's part of the P row (bf16, MN-major, swizzled: the B operand of the PV
+//     product) and keeps its share of every row sum;
 //   * warps 8-11 (epilogue) add the row-sum shares, read O^T from TMEM and write the normalised
 //     output or, for a split item, the (O, m, l) partials; the last chunk of a split
 //     (request, head, row group) to finish merges all its chunks.  This runs while the softmax
 //     warps are already on the next item.
 // Every mbarrier wait is bounded in time; an expired wait records WISP_DEV_TIMEOUT and the CTA
-// drains.  No named barrier is used: a warp that gives up cannot leave the others blocked.
+// drains.  No named barrier is used: a warp that gives up cannot leave the others blocked, and the
+// TMEM is freed once every warp has arrived on a final mbarrier.
 #include "attn.cuh"
 #include "sm100_ptx.cuh"
 
