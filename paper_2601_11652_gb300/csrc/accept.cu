@@ -361,6 +361,9 @@ __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ Acce
   __shared__ int s_owner, s_take_last;
   __shared__ ff s_thr;
 
+  // launched as a programmatic dependent of the kernel before it: nothing is read before that
+  // grid has completed and its writes are visible
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   cg::cluster_group cluster = cg::this_cluster();
   const int C = p.cluster;
   const int rank = (int)cluster.block_rank();
@@ -864,13 +867,17 @@ cudaError_t walk_t(const AcceptParams &ap, cudaStream_t s) {
   const bool tab = std::is_same<LT, uint16_t>::value && ap.V >= kExpTabMinV;
   cfg.dynamicSmemBytes = (size_t)rounds * NW * sizeof(ff) + (tab ? kExpTabSize * sizeof(ff) : 0);
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = (unsigned)ap.cluster;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  // programmatic dependent launch: the clusters may be placed while the previous kernel's last
+  // CTAs run (the kernel waits for it before it reads anything)
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, accept_kernel<LT>, ap);
 }
 

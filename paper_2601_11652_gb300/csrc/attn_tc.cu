@@ -358,7 +358,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::mbar_arrive(B.it_full + slot);
       }
       it = __shfl_sync(0xffffffffu, it, 0);
-      if (it < 0) break;
+      if (it < 0) {
+        // no item left for this CTA: a kernel launched after this one as a programmatic
+        // dependent (the acceptance walk) may be scheduled; it still waits for this grid to finish
+        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+        break;
+      }
       const WorkItem w = p.items[it];
       const int qb = li & 1;
       if (!wait_bar(B.q_empty + qb, ((li >> 1) & 1) ^ 1, s_abort)) { ok = false; break; }
