@@ -74,11 +74,20 @@ def _peaks():
         return 6800.0, "fallback"
 
 
-def _kernel_sha() -> str:
+# the sources each profiled kernel is built from (its launch set-up in api.cu included)
+KERNEL_SOURCES = {
+    "attention": ("api.cu", "attn.cuh", "attn_tc.cu", "common.cuh", "plan.cu", "plan.cuh", "sm100_ptx.cuh"),
+    "accept": ("accept.cu", "accept.cuh", "api.cu", "common.cuh"),
+}
+
+
+def _kernel_sha(kernel: str = None) -> str:
+    """sha256 (16 hex digits) of the kernel's sources, or of every csrc/*.cu, *.cuh if kernel is None."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2601_11652_gb300", "csrc")
+    want = KERNEL_SOURCES.get(kernel)
     for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh")):
+        if name.endswith((".cu", ".cuh")) and (want is None or name in want):
             with open(os.path.join(csrc, name), "rb") as f:
                 h.update(name.encode() + f.read())
     return h.hexdigest()[:16]
@@ -93,7 +102,7 @@ def _profile_traffic(kernel: str, workload: str):
         return None
     sha = re.search(r"kernel_source_sha:\s*(\w+)", text)
     tr = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
-    if not sha or not tr or sha.group(1) != _kernel_sha():
+    if not sha or not tr or sha.group(1) != _kernel_sha(kernel):
         return None
     return float(tr.group(1))
 

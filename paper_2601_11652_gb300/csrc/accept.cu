@@ -36,6 +36,11 @@ namespace {
 
 constexpr int NW = kAcceptThreads / 32;
 constexpr int NT = kAcceptThreads;
+// vectors (normaliser passes) and rounds (draw sweep) a thread keeps loaded ahead of the one it
+// uses, in a ring of registers with one copy of the loop body: with one 16-byte load in flight per
+// thread the streams of accept_kernel are latency-bound
+constexpr int kZAhead = 8;
+constexpr int kSweepAhead = 4;
 
 template <typename LT>
 struct LTraits;
@@ -152,6 +157,26 @@ __device__ __forceinline__ ff elem_exp<uint16_t>(const uint4 &w, int i, float m,
   const int idx = exp_tab_index((i & 1) ? (u >> 16) : (u & 0xFFFFu));
   if (tab && idx >= 0) return tab[idx];
   return exp_direct(vec_elem<uint16_t>(w, i), m, th, tl);
+}
+
+// Sum of two non-negative double-float values: Dekker's addition without the TwoSum of the low
+// parts.  With operands of one sign no cancellation occurs and the relative error stays within
+// about 3 * 2^-48 (the full ff_add is kept wherever a difference is formed).
+__device__ __forceinline__ ff ff_add_pos(ff a, ff b) {
+  ff s = ff_two_sum(a.hi, b.hi);
+  s.lo = __fadd_rn(s.lo, __fadd_rn(a.lo, b.lo));
+  return ff_fast_two_sum(s.hi, s.lo);
+}
+
+// Pairwise sum of the E non-negative terms of one vector (three levels for E = 8).
+template <int E>
+__device__ __forceinline__ ff ff_tree_pos(ff (&t)[E]) {
+#pragma unroll
+  for (int w = 1; w < E; w <<= 1) {
+#pragma unroll
+    for (int i = 0; i < E; i += 2 * w) t[i] = ff_add_pos(t[i], t[i + w]);
+  }
+  return t[0];
 }
 
 // Draw weight from e = exp(z - m): e itself, or the residual max(0, e - q Z) (as draw_weight).
@@ -346,7 +371,7 @@ __global__ void __launch_bounds__(NT) row_stats_kernel(const __grid_constant__ A
 }
 
 template <typename LT>
-__global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ AcceptParams p) {
+__global__ void __launch_bounds__(NT, 2) accept_kernel(const __grid_constant__ AcceptParams p) {
   constexpr int E = LTraits<LT>::E;
   extern __shared__ ff s_tile[];  // [rounds * NW] per-(round, warp) draw sums, then the exp table (bf16)
   __shared__ float s_th[256], s_tl[256];
@@ -422,18 +447,36 @@ __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ Acce
     xslot ^= 1;
     return t;
   };
+  // double-float sum of f(element) over this thread's vectors of a row, in vector order; w[u] holds
+  // the vector u rounds ahead of the current one
+  auto thread_sum = [&](const LT *row, auto &&f) -> ff {
+    ff acc = {0.0f, 0.0f};
+    uint4 w[kZAhead];
+#pragma unroll
+    for (int u = 0; u < kZAhead; ++u) {
+      const int64_t vi = vlo + tid + (int64_t)u * NT;
+      if (vi < vhi) w[u] = load_vec<LT>(row, vi, V, vec_z);
+    }
+#pragma unroll 1
+    for (int64_t vi = vlo + tid; vi < vhi; vi += NT) {
+      const uint4 cur = w[0];
+#pragma unroll
+      for (int u = 0; u + 1 < kZAhead; ++u) w[u] = w[u + 1];
+      const int64_t vn = vi + (int64_t)kZAhead * NT;
+      if (vn < vhi) w[kZAhead - 1] = load_vec<LT>(row, vn, V, vec_z);
+      ff t[E];
+#pragma unroll
+      for (int i = 0; i < E; ++i) t[i] = f(cur, i);
+      acc = ff_add_pos(acc, ff_tree_pos<E>(t));
+    }
+    return acc;
+  };
   // double-float normaliser of a row (re-streamed); m is the row's exact max
   auto row_Zff = [&](const LT *row, float m) -> ff {
-    ff acc = {0.0f, 0.0f};
-    for (int64_t vi = vlo + tid; vi < vhi; vi += NT) {
-      const uint4 w = load_vec<LT>(row, vi, V, vec_z);
-#pragma unroll
-      for (int i = 0; i < E; ++i) {
-        const ff x = ff_two_sum(vec_elem<LT>(w, i), -m);
-        acc = ff_add(acc, ff_exp_nonpos(x.hi, x.lo, s_th, s_tl));
-      }
-    }
-    return cluster_total(acc);
+    return cluster_total(thread_sum(row, [&](const uint4 &w, int i) {
+      const ff x = ff_two_sum(vec_elem<LT>(w, i), -m);
+      return ff_exp_nonpos(x.hi, x.lo, s_th, s_tl);
+    }));
   };
 
   // ---- the in-order walk (Eq. 1-2) -------------------------------------------
@@ -563,43 +606,59 @@ __global__ void __launch_bounds__(NT) accept_kernel(const __grid_constant__ Acce
   // (only for rows much longer than the table)
   ff *s_etab = std::is_same<LT, uint16_t>::value && V >= kExpTabMinV ? s_tile + rounds * NW : nullptr;
   if (s_etab) {
+#pragma unroll 2
     for (int idx = tid; idx < kExpTabSize; idx += NT) {
       const float u = bf16_bits_to_float(exp_tab_bits(idx));
       s_etab[idx] = u > m ? ff{0.0f, 0.0f} : draw_weight(u, m, false, 0.0f, ff{}, s_th, s_tl);  // u > m never occurs
     }
     __syncthreads();
   }
-  if (residual && !have_Zff) {
-    ff acc = {0.0f, 0.0f};
-    for (int64_t vi = vlo + tid; vi < vhi; vi += NT) {
-      const uint4 w = load_vec<LT>(row, vi, V, vec_z);
-#pragma unroll
-      for (int i = 0; i < E; ++i) acc = ff_add(acc, elem_exp<LT>(w, i, m, s_etab, s_th, s_tl));
-    }
-    Zff = cluster_total(acc);
-  }
+  if (residual && !have_Zff)
+    Zff = cluster_total(thread_sum(row, [&](const uint4 &w, int i) { return elem_exp<LT>(w, i, m, s_etab, s_th, s_tl); }));
   ff S = {0.0f, 0.0f};
   for (;;) {
     ff run = {0.0f, 0.0f};
+    // the row's and the draft's vectors of round rd + u in w[u], q[u]
+    uint4 w[kSweepAhead];
+    float q[kSweepAhead][E];
+    auto load_round = [&](int rd, uint4 &wv, float (&qv)[E]) {
+      const int64_t vi = vlo + (int64_t)rd * NT + tid;
+      if (rd < rounds && vi < vhi) {
+        wv = load_vec<LT>(row, vi, V, vec_z);
+        if (residual) {
+          load_q<E>(qrow, vi * E, V, vec_q, qv);
+        } else {
+#pragma unroll
+          for (int i = 0; i < E; ++i) qv[i] = 0.0f;
+        }
+      }
+    };
+#pragma unroll
+    for (int u = 0; u < kSweepAhead; ++u) load_round(u, w[u], q[u]);
+#pragma unroll 1
     for (int rd = 0; rd < rounds; ++rd) {
+      const uint4 cw = w[0];
+      float cq[E];
+#pragma unroll
+      for (int i = 0; i < E; ++i) cq[i] = q[0][i];
+#pragma unroll
+      for (int u = 0; u + 1 < kSweepAhead; ++u) {
+        w[u] = w[u + 1];
+#pragma unroll
+        for (int i = 0; i < E; ++i) q[u][i] = q[u + 1][i];
+      }
+      load_round(rd + kSweepAhead, w[kSweepAhead - 1], q[kSweepAhead - 1]);
       const int64_t vi = vlo + (int64_t)rd * NT + tid;
       ff part = {0.0f, 0.0f};
       if (vi < vhi) {
-        const uint4 w = load_vec<LT>(row, vi, V, vec_z);
-        float q[E];
-        if (residual) {
-          load_q<E>(qrow, vi * E, V, vec_q, q);
-        } else {
+        ff t[E];
 #pragma unroll
-          for (int i = 0; i < E; ++i) q[i] = 0.0f;
-        }
-#pragma unroll
-        for (int i = 0; i < E; ++i)
-          part = ff_add(part, weight_from(elem_exp<LT>(w, i, m, s_etab, s_th, s_tl), residual, q[i], Zff));
+        for (int i = 0; i < E; ++i) t[i] = weight_from(elem_exp<LT>(cw, i, m, s_etab, s_th, s_tl), residual, cq[i], Zff);
+        part = ff_tree_pos<E>(t);
       }
-      for (int o = 16; o > 0; o >>= 1) part = ff_add(part, ff_shfl_xor(part, o));
+      for (int o = 16; o > 0; o >>= 1) part = ff_add_pos(part, ff_shfl_xor(part, o));
       if (lane == 0) s_tile[rd * NW + warp] = part;
-      run = ff_add(run, part);
+      run = ff_add_pos(run, part);
     }
     // run is the warp's sum over all rounds (same value in every lane): count it once
     if (lane != 0) run = {0.0f, 0.0f};
@@ -763,14 +822,23 @@ __global__ void __launch_bounds__(NT) row_argmax_kernel(const __grid_constant__ 
   float m = -INFINITY;
   int idx = INT32_MAX;
   // a lane visits its elements in increasing token order, so a strict ">" keeps the first maximum
-  for (int64_t vi = vlo + lane; vi < vhi; vi += 32) {
-    const uint4 w = load_vec<LT>(rowp, vi, V, p.vec_z != 0);
+  // (the loads of 4 vectors in flight together)
+  for (int64_t v0 = vlo + lane; v0 < vhi; v0 += 4 * 32) {
+    uint4 w[4];
 #pragma unroll
-    for (int i = 0; i < E; ++i) {
-      const float z = vec_elem<LT>(w, i);
-      if (z > m) {
-        m = z;
-        idx = (int)(vi * E + i);
+    for (int u = 0; u < 4; ++u)
+      if (v0 + u * 32 < vhi) w[u] = load_vec<LT>(rowp, v0 + u * 32, V, p.vec_z != 0);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t vi = v0 + u * 32;
+      if (vi >= vhi) break;
+#pragma unroll
+      for (int i = 0; i < E; ++i) {
+        const float z = vec_elem<LT>(w[u], i);
+        if (z > m) {
+          m = z;
+          idx = (int)(vi * E + i);
+        }
       }
     }
   }

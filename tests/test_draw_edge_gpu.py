@@ -10,7 +10,7 @@ import torch
 
 import oracle
 from paper_2601_11652_gb300 import workload as wl
-from tests.gpu_util import SAMPLE_WINDOW
+from tests.gpu_util import SAMPLE_WINDOW, compare_accept
 
 pytestmark = pytest.mark.gpu
 
@@ -79,3 +79,23 @@ def test_draw_next_to_a_cdf_edge_matches_the_oracle(seed, V):
     for r in near:
         assert got["accepted_len"][r] == ref["accepted_len"][r]
         assert got["next_token"][r] == ref["next_token"][r], (r, float(ref["sample_margin"][r]))
+
+
+@pytest.mark.parametrize("shift", [-40.0, 45.0, 75.0])
+def test_draw_with_shifted_logits_matches_the_oracle(shift):
+    """Row maxima far below 0, near 55 and above the exp table's range (|u| < 64): the table entries
+    exp(u - m) reach the float underflow range, or most elements take the direct exp; all must give
+    the oracle's tokens."""
+    from paper_2601_11652_gb300.device_batch import DeviceBatch
+    b = wl.make_small_batch(13, B=12, Hq=8, Hkv=2, D=128, V=40000, dtype="bf16", k_range=(2, 7), ctx_range=(0, 200))
+    b.logits = wl.f32_to_bf16_bits(wl.bf16_bits_to_f32(b.logits) + np.float32(shift))
+    ref = oracle.accept(b)
+    assert np.any(ref["accepted_len"] < b.draft_lens), "some request draws from a residual"
+    db = DeviceBatch.from_host(b)
+    db.step()
+    torch.cuda.synchronize()
+    code, rid = db.device_status()
+    assert code == 0, (code, rid)
+    got = db.results()
+    n, _ = compare_accept(b, got["accepted_len"], got["next_token"], ref)
+    assert n >= b.B - 2
