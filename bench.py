@@ -143,8 +143,13 @@ class ClockSampler:
         except Exception:
             self.proc.kill()
         self.f.close()
+        return self.summarise(self.path)
+
+    @staticmethod
+    def summarise(path: str):
+        """Median SM clock, max clock and the throttle reasons seen in a sample file."""
         rows = []
-        for line in open(self.path):
+        for line in open(path):
             parts = [p.strip() for p in line.split(",")]
             if len(parts) < 9:
                 continue

@@ -1,0 +1,85 @@
+"""CPU: the host-side arithmetic of bench.py -- algorithmic bytes, the per-kernel source hashes
+that decide whether a committed ncu summary still describes the sources, and the clock summary."""
+import os
+import shutil
+
+import numpy as np
+
+import bench
+from paper_2601_11652_gb300 import workload as wl
+
+
+def test_attention_bytes_counts_every_visible_token_once():
+    b = wl.make_small_batch(3, B=4, Hq=8, Hkv=2, D=64, V=512, dtype="bf16", k_range=(0, 5), ctx_range=(0, 90))
+    kv = qo = bt = 0
+    for r in range(b.B):
+        n = int(b.context_lens[r]) + int(b.draft_lens[r]) + 1
+        kv += n * b.Hkv * b.D * 2 * 2          # K and V, bf16
+        qo += (int(b.draft_lens[r]) + 1) * b.Hq * b.D * 2 * 2
+        bt += -(-n // 16) * 4
+    assert bench.attention_bytes(b) == kv + qo + bt
+
+
+def test_accept_bytes_rows_up_to_the_rejection_and_one_draft_row():
+    b = wl.make_small_batch(4, B=3, Hq=4, Hkv=4, D=64, V=1000, dtype="f32", k_range=(3, 3), ctx_range=(0, 10))
+    L = [0, 3, 1]  # rejection at 0, all accepted, rejection at 1
+    rows = (1 + 4 + 2) * 1000 * 4
+    qrow = 2 * 1000 * 4
+    decisions = 1 + 3 + 2
+    assert bench.accept_bytes(b, L) == rows + qrow + decisions * 72 + 3 * 16
+
+
+def _copy_sources(tmp_path):
+    root = tmp_path / "repo"
+    shutil.copytree(os.path.join(bench.ROOT, "paper_2601_11652_gb300", "csrc"),
+                    root / "paper_2601_11652_gb300" / "csrc")
+    return root
+
+
+def test_kernel_sources_exist():
+    csrc = os.path.join(bench.ROOT, "paper_2601_11652_gb300", "csrc")
+    for kernel, files in bench.KERNEL_SOURCES.items():
+        for f in files:
+            assert os.path.isfile(os.path.join(csrc, f)), (kernel, f)
+
+
+def test_kernel_hash_follows_only_its_own_sources(tmp_path, monkeypatch):
+    root = _copy_sources(tmp_path)
+    monkeypatch.setattr(bench, "ROOT", str(root))
+    before = {k: bench._kernel_sha(k) for k in (None, "attention", "accept")}
+    with open(root / "paper_2601_11652_gb300" / "csrc" / "accept.cu", "a") as f:
+        f.write("\n// edit\n")
+    after = {k: bench._kernel_sha(k) for k in (None, "attention", "accept")}
+    assert after["attention"] == before["attention"]
+    assert after["accept"] != before["accept"]
+    assert after[None] != before[None]
+    with open(root / "paper_2601_11652_gb300" / "csrc" / "common.cuh", "a") as f:
+        f.write("\n// shared header\n")
+    assert bench._kernel_sha("attention") != before["attention"]
+
+
+def test_profile_traffic_only_while_the_sources_match(tmp_path, monkeypatch):
+    root = _copy_sources(tmp_path)
+    monkeypatch.setattr(bench, "ROOT", str(root))
+    (root / "profiles").mkdir()
+    prof = root / "profiles" / "accept_demo.md"
+    prof.write_text(f"kernel_source_sha: {bench._kernel_sha('accept')}  (note)\n\ndram_bytes_per_launch: 12345\n")
+    assert bench._profile_traffic("accept", "demo") == 12345.0
+    assert bench._profile_traffic("attention", "demo") is None  # no such file
+    with open(root / "paper_2601_11652_gb300" / "csrc" / "accept.cuh", "a") as f:
+        f.write("\n")
+    assert bench._profile_traffic("accept", "demo") is None
+
+
+def test_clock_summary(tmp_path):
+    p = tmp_path / "clocks.csv"
+    na, act = "Not Active", "Active"
+    lines = [f"0, {mhz}, 2070, 900.0, 0x0, {na}, {na}, {na}, {cap}" for mhz, cap in
+             [(2070, na), (1980, act), (2010, na), (1500, na), (2070, na)]]
+    p.write_text("\n".join(lines + ["garbage line", "0, [N/A], 2070, 1, 0x0, a, b, c, d"]) + "\n")
+    s = bench.ClockSampler.summarise(str(p))
+    assert s == {"sm_mhz": 2010.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 5}
+    empty = tmp_path / "empty.csv"
+    empty.write_text("")
+    assert bench.ClockSampler.summarise(str(empty)) is None
+    assert np.isfinite(s["sm_mhz"])
