@@ -108,6 +108,33 @@ def _profile_traffic(kernel: str, workload: str):
     return float(tr.group(1))
 
 
+def _profile_inst(kernel: str, workload: str):
+    """Warp instructions per launch summed over the kernels of the committed ncu summary of
+    `kernel`, if it matches this source (None otherwise)."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    sha = re.search(r"kernel_source_sha:\s*(\w+)", text)
+    inst = re.findall(r"\|\s*smsp__inst_executed\.sum\s*\|\s*([0-9.eE+]+)\s*inst", text)
+    if not sha or not inst or sha.group(1) != _kernel_sha(kernel):
+        return None
+    return float(sum(float(x) for x in inst))
+
+
+def issue_roofline(warp_inst: float, ms: float, sms: int, sm_mhz: float):
+    """Instruction-issue view of a kernel group bound by arithmetic and barriers rather than bytes:
+    warp instructions per second against the issue peak, sms x 4 schedulers x 1 warp instruction
+    per clock at the given SM clock."""
+    if not warp_inst or not ms or not sms or not sm_mhz:
+        return None
+    achieved = warp_inst / (ms * 1e-3) / 1e9
+    peak = sms * 4 * sm_mhz * 1e6 / 1e9
+    return {"bound": "issue", "achieved": achieved, "peak": peak, "unit": "G warp-inst/s",
+            "frac": achieved / peak, "warp_inst_per_launch": warp_inst}
+
+
 # --------------------------------------------------------------------------
 # clocks during the timed region
 # --------------------------------------------------------------------------
@@ -314,6 +341,12 @@ def run_ours(args, batch, rank, world, local_rank):
 
     # end to end: per-step inputs from pinned host memory, results back to the host
     e2e = _e2e(db, batch, args, flush, torch, verified)
+    try:
+        acc_issue = issue_roofline(_profile_inst("accept", batch.name), acc_ms,
+                                   torch.cuda.get_device_properties(dev).multi_processor_count,
+                                   clocks["sm_max_mhz"] if clocks else None)
+    except Exception:
+        acc_issue = None
 
     if rank != 0:
         return
@@ -326,7 +359,8 @@ def run_ours(args, batch, rank, world, local_rank):
                          "algorithmic_bytes_per_launch": ab},
             "accept_roofline": {"bound": "hbm", "achieved": acc_gbs, "peak": peak, "unit": "GB/s",
                                 "frac": acc_gbs / peak, "algorithmic_bytes_per_launch": cb,
-                                "traffic": _profile_traffic("accept", batch.name)},
+                                "traffic": _profile_traffic("accept", batch.name),
+                                "issue": acc_issue},
             "step_algorithmic_gbs": (ab + cb) / (ms_per_step * 1e-3) / 1e9,
             "emitted_tokens_per_s": (verified_all + batch.B * world) / (ms_per_step / 1e3),
             "mean_acceptance": float(verified / max(1, batch.total_draft)),

@@ -83,3 +83,22 @@ def test_clock_summary(tmp_path):
     empty.write_text("")
     assert bench.ClockSampler.summarise(str(empty)) is None
     assert np.isfinite(s["sm_mhz"])
+
+
+def test_issue_roofline_from_the_profile(tmp_path, monkeypatch):
+    root = _copy_sources(tmp_path)
+    monkeypatch.setattr(bench, "ROOT", str(root))
+    (root / "profiles").mkdir()
+    prof = root / "profiles" / "accept_demo.md"
+    prof.write_text(f"kernel_source_sha: {bench._kernel_sha('accept')}\n\n"
+                    "| smsp__inst_executed.sum | 1000000.000000 inst |\n"
+                    "| smsp__inst_executed.sum | 3000000.000000 inst |\n")
+    w = bench._profile_inst("accept", "demo")
+    assert w == 4.0e6
+    r = bench.issue_roofline(w, 0.01, 100, 2000.0)  # 4e6 warp instructions in 10 us on 100 SMs at 2 GHz
+    assert abs(r["achieved"] - 400.0) < 1e-9 and abs(r["peak"] - 800.0) < 1e-9 and abs(r["frac"] - 0.5) < 1e-12
+    assert bench.issue_roofline(None, 0.01, 100, 2000.0) is None
+    assert bench.issue_roofline(w, 0.01, 100, None) is None
+    with open(root / "paper_2601_11652_gb300" / "csrc" / "accept.cu", "a") as f:
+        f.write("\n")
+    assert bench._profile_inst("accept", "demo") is None
