@@ -89,3 +89,26 @@ def test_bad_input_is_reported_and_the_rest_is_exact(oracle_mod, dtype, kind):
         # as the oracle does (a row with no finite logit has no softmax; the oracle leaves that
         # undefined case unflagged, the library reports it)
         assert oracle_mod.accept(b, check=False)["status"][r] == ORACLE_STATUS[code]
+
+
+def test_too_many_query_rows_per_kv_head_is_reported(oracle_mod):
+    """g (k + 1) = 4 x 33 = 132 query rows of one KV head, above the library's 128: the planner flags
+    the request WISP_DEV_UNSUPPORTED and the step runs every other request exactly."""
+    from paper_2601_11652_gb300.device_batch import DeviceBatch
+    k = np.array([3, 2, 32, 4, 1], np.int32)
+    c = np.array([100, 50, 80, 300, 10], np.int32)
+    b = wl.make_batch_from_lengths("rows132", draft_lens=k, context_lens=c, Hq=8, Hkv=2, D=128, V=3000,
+                                   dtype="bf16", sigma=float(wl.sigma_for_alpha(0.7)), key=(140, 0))
+    ref_attn = oracle_mod.attention(b)
+    ref_acc = oracle_mod.accept(b)
+    db = DeviceBatch.from_host(b)
+    db.step()
+    torch.cuda.synchronize()
+    assert db.device_status() == (5, int(b.request_ids[2]))  # WISP_DEV_UNSUPPORTED
+    got = db.results()
+    others = [0, 1, 3, 4]
+    rows = subset_rows(b, others)
+    assert attn_max_err(got["out"][rows], ref_attn[rows]) <= ATTN_TOL["bf16"]
+    for i in others:
+        assert got["accepted_len"][i] == ref_acc["accepted_len"][i], i
+        assert got["next_token"][i] == ref_acc["next_token"][i], i
