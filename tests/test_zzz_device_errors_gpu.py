@@ -112,3 +112,28 @@ def test_too_many_query_rows_per_kv_head_is_reported(oracle_mod):
     for i in others:
         assert got["accepted_len"][i] == ref_acc["accepted_len"][i], i
         assert got["next_token"][i] == ref_acc["next_token"][i], i
+
+
+def test_empty_batch_is_a_no_op():
+    """B = 0: every entry point accepts the empty batch (attention pointers may be NULL), enqueues
+    only the planner, reports no error and writes no output."""
+    from paper_2601_11652_gb300 import binding as wb
+    dev = "cuda"
+    lens = torch.zeros(1, dtype=torch.int32, device=dev)
+    logits = torch.zeros((1, 1000), dtype=torch.bfloat16, device=dev)
+    su = torch.zeros(1, dtype=torch.float32, device=dev)
+    out_L = torch.full((1,), -7, dtype=torch.int32, device=dev)
+    out_t = torch.full((1,), -7, dtype=torch.int32, device=dev)
+    a = wb.wisp_attn_args()
+    a.B, a.Hq, a.Hkv, a.D, a.block_size, a.qkv_dtype = 0, 8, 2, 128, 16, wb.WISP_BF16
+    c = wb.wisp_accept_args()
+    c.B, c.V, c.total_q_rows, c.total_draft, c.logits_dtype = 0, 1000, 0, 0, wb.WISP_BF16
+    c.draft_lens, c.target_logits, c.sample_uniforms = lens.data_ptr(), logits.data_ptr(), su.data_ptr()
+    c.accepted_len, c.next_token = out_L.data_ptr(), out_t.data_ptr()
+    ws = wb.alloc_workspace(wb.wisp_verify_workspace_size(a, c), dev)
+    wb.wisp_verify_step(a, c, ws)
+    wb.wisp_verify_attention(a, ws)
+    wb.wisp_verify_accept(c, ws)
+    torch.cuda.synchronize()
+    assert wb.wisp_verify_get_device_status(ws) == (0, 0)
+    assert out_L.item() == -7 and out_t.item() == -7
