@@ -140,8 +140,10 @@ int oracle_attention(int B, int Hq, int Hkv, int D, int bs, int max_blocks, int 
 /* Acceptance and the target token                                          */
 /* ------------------------------------------------------------------------ */
 
-/* p(v) = exp(z_v - max z) / sum_w exp(z_w - max z) for one logit row. */
-void oracle_row_softmax(int V, int dtype, const void *row, double *p) {
+/* p(v) = exp(z_v - max z) / sum_w exp(z_w - max z) for one logit row.  Returns 0 when the
+ * softmax is undefined: no finite maximum (every logit -inf, or a +inf one) or a normaliser that
+ * is not a finite positive number (a NaN logit); p is then not meaningful. */
+static int row_softmax_checked(int V, int dtype, const void *row, double *p) {
     double mx = -INFINITY;
     for (int v = 0; v < V; ++v) {
         double z = elem(row, dtype, v);
@@ -153,6 +155,11 @@ void oracle_row_softmax(int V, int dtype, const void *row, double *p) {
         Z += p[v];
     }
     for (int v = 0; v < V; ++v) p[v] /= Z;
+    return isfinite(mx) && Z > 0.0 && isfinite(Z);
+}
+
+void oracle_row_softmax(int V, int dtype, const void *row, double *p) {
+    (void)row_softmax_checked(V, dtype, row, p);
 }
 
 /*
@@ -218,14 +225,22 @@ int oracle_accept(int B, int V, const int32_t *draft_lens, int dtype, const void
         double *w = (double *)malloc(sizeof(double) * (size_t)V);
         int st = OR_OK, L = k;
         double amargin = INFINITY;
+        /* a draft token outside [0, V) anywhere in the draft makes the request invalid */
+        for (int j = 0; j < k; ++j) {
+            const int32_t y = draft_tokens[d0[r] + j];
+            if (y < 0 || y >= V) { st = OR_BAD_TOKEN; break; }
+        }
         /* Eq. 1-2: walk the draft in order, stop at the first rejection */
-        for (int j = 1; j <= k; ++j) {
+        for (int j = 1; j <= k && st == OR_OK; ++j) {
             const int64_t drow = d0[r] + j - 1;
             const int32_t y = draft_tokens[drow];
             if (y < 0 || y >= V) { st = OR_BAD_TOKEN; break; }
             const double qy = (double)draft_probs[drow * V + y];
             if (!(qy >= 0.0)) { st = OR_BAD_PROB; break; }
-            oracle_row_softmax(V, dtype, (const char *)logits + (size_t)(row0[r] + j - 1) * V * esz, p);
+            if (!row_softmax_checked(V, dtype, (const char *)logits + (size_t)(row0[r] + j - 1) * V * esz, p)) {
+                st = OR_BAD_PROB;
+                break;
+            }
             const double a = (qy == 0.0) ? 1.0 : fmin(1.0, p[y] / qy);
             const double u = (double)accept_u[drow];
             const double gap = fabs(u - a);
@@ -236,7 +251,10 @@ int oracle_accept(int B, int V, const int32_t *draft_lens, int dtype, const void
         double smargin = 0.0;
         if (st == OR_OK) {
             /* Eq. 3 at the stopping position: residual on rejection, p after a full accept */
-            oracle_row_softmax(V, dtype, (const char *)logits + (size_t)(row0[r] + L) * V * esz, p);
+            if (!row_softmax_checked(V, dtype, (const char *)logits + (size_t)(row0[r] + L) * V * esz, p))
+                st = OR_BAD_PROB;
+        }
+        if (st == OR_OK) {
             if (L < k) {
                 const float *qrow = draft_probs + (size_t)(d0[r] + L) * V;
                 for (int v = 0; v < V; ++v) {

@@ -178,3 +178,35 @@ def test_rejects_out_of_range_token(oracle_mod):
         oracle_mod.accept(b)
     out = oracle_mod.accept(b, check=False)
     assert out["status"][0] == 4 and out["accepted_len"][0] == -1
+
+
+def test_undefined_softmax_rows_are_flagged(oracle_mod):
+    """A logit row the rule reads must have a softmax: every logit -inf, a +inf or a NaN logit
+    flags the request (status bad_prob = 5); a -inf entry among finite ones is an ordinary zero
+    probability.  The other request of the batch is unaffected."""
+    ninf, pinf, nan = -np.inf, np.inf, np.nan
+    fine = [0.0, 1.0, -1.0, 0.5]
+    for bad_row in ([ninf] * 4, [0.0, pinf, 1.0, 2.0], [0.0, nan, 1.0, 2.0]):
+        # request 0: one draft token, rows 0 (decision) and 1; request 1: k = 0, one row
+        b = _Batch([bad_row, fine, fine], [1, 0], [2], [[0.25] * 4], [0.1], [0.3, 0.6])
+        out = oracle_mod.accept(b, check=False)
+        assert out["status"].tolist() == [5, 0], bad_row
+        assert out["accepted_len"][0] == -1 and out["next_token"][0] == -1
+        ref = oracle_mod.accept(_Batch([fine], [0], [], [], [], [0.6]))
+        assert out["next_token"][1] == ref["next_token"][0]
+    # the draw row (row L) is read too: after a full acceptance the bonus row is all -inf
+    b = _Batch([fine, [ninf] * 4], [1], [1], [[0.25] * 4], [0.0], [0.5])
+    assert oracle_mod.accept(b, check=False)["status"][0] == 5
+    # -inf among finite logits: p = 0 there, never drawn
+    masked = [ninf, 1.0, ninf, 1.0]
+    out = oracle_mod.accept(_Batch([masked], [0], [], [], [], [0.99]))
+    assert out["status"][0] == 0 and out["next_token"][0] == 3
+
+
+def test_out_of_range_token_anywhere_in_the_draft_is_flagged(oracle_mod):
+    """The whole draft is validated, also a token after the first rejection (status bad_token = 4)."""
+    rows = [[0.0, 0.0, 0.0, 0.0]] * 3
+    # token 0 has p = 0.25 against q = 1.0: rejected with u = 0.9; token 1 is out of range
+    b = _Batch(rows, [2], [0, 9], [[1.0, 0.0, 0.0, 0.0], [0.25] * 4], [0.9, 0.1], [0.5])
+    out = oracle_mod.accept(b, check=False)
+    assert out["status"][0] == 4 and out["accepted_len"][0] == -1
