@@ -74,9 +74,10 @@ typedef enum {
   WISP_DEV_BAD_LENGTH = 1,   /* k_r < 0, c_r < 0, c_r + k_r + 1 > max_blocks_per_seq * block_size,
                                 or sum of lengths disagrees with total_q_rows / total_draft */
   WISP_DEV_BAD_BLOCK = 2,    /* a block id needed by the request is outside [0, num_blocks) */
-  WISP_DEV_BAD_TOKEN = 3,    /* a draft token outside [0, V) */
-  WISP_DEV_BAD_PROB = 4,     /* a draft probability q(y) that is negative or NaN, or a logit row
-                                with no finite maximum / non-finite normaliser */
+  WISP_DEV_BAD_TOKEN = 3,    /* a draft token outside [0, V), anywhere in the draft */
+  WISP_DEV_BAD_PROB = 4,     /* a draft probability q(y) that is negative or NaN at a decision the
+                                walk takes, or a logit row it reads (rows 0..L) with no finite
+                                maximum / no finite positive normaliser (a row without a softmax) */
   WISP_DEV_UNSUPPORTED = 5,  /* (Hq / Hkv) * (k_r + 1) > 128 query rows, or k_r > 1024 */
   WISP_DEV_TIMEOUT = 6,      /* a bounded device-side wait gave up (no kernel waits unboundedly) */
   WISP_DEV_NO_BLOCKS = 7     /* (wisp_kv.h) the free page pool could not serve the request */
