@@ -11,8 +11,6 @@ those the step could use return to the stack in table order.  Written as loops o
 """
 from __future__ import annotations
 
-import numpy as np
-
 PAGE = 16
 OK, BAD_LENGTH, BAD_BLOCK, NO_BLOCKS = 0, 1, 2, 7
 

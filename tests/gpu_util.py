@@ -1,8 +1,6 @@
 """Helpers shared by the GPU parity tests: tolerances and the oracle comparison."""
 import numpy as np
 
-from paper_2601_11652_gb300 import workload as wl
-
 # attention: max abs error of the output (bf16 KV + fp32 accumulate; fp32 inputs)
 ATTN_TOL = {"bf16": 2e-2, "f32": 1e-4}
 # acceptance decisions within this distance of their threshold are logged, not failed

@@ -3,7 +3,6 @@ and verified tokens (sum); each rank's batch is its own replica, so nothing else
 import os
 import socket
 
-import pytest
 import torch.multiprocessing as mp
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
