@@ -22,6 +22,7 @@
 // memory, summed in rank order so every CTA holds bit-identical values); the CTA holding the
 // crossing of u * total scans its tiles, then one warp scans the tile, then one lane its
 // elements.
+#include <cfloat>
 #include <cooperative_groups.h>
 #include <cstring>
 #include <type_traits>
@@ -532,11 +533,22 @@ __global__ void __launch_bounds__(NT, 2) accept_kernel(const __grid_constant__ A
             break;
           }
           if (d.qy == 0.0f) continue;  // a = 1: accepted
+          if (!(d.zy > -INFINITY)) {  // a masked token: p(y) = 0 exactly, accepted only if u = 0
+            if (d.u <= 0.0f) continue;
+            state = 2;
+            break;
+          }
           // certified relative error of Z (see RowStats) and of the ratio p(y)/q(y)
           // terms: one exp error per element and per rescale on its way (thread, CTA, row), three
           // roundings in the argument (z - m, log2 e, the product) of every element and every
           // rescale, the 32-term pairwise sums; the decision's own exp and ratio on top
           const float x = d.zy - mi;
+          // outside the range of the fp32 ratio (2^x flushes to zero below 2^-126, a subnormal q(y)
+          // loses bits): decide in double precision
+          if (x * kLog2e < -126.0f || d.qy < FLT_MIN) {
+            state = 4;
+            break;
+          }
           const float dz = 1.05f * ((float)(rs.nres + 2) * kEx2RelErr + 3.0f * 0x1p-24f * (mi - rs.mfirst) +
                                     3.0f * 0x1p-24f * (rs.A / Z.hi) + 6.0f * 0x1p-24f) +
                            1e-12f;
@@ -568,9 +580,9 @@ __global__ void __launch_bounds__(NT, 2) accept_kernel(const __grid_constant__ A
         const ff zf = row_Zff(logits + (Q0 + i) * (int64_t)V, mi);
         if (tid == 0) {
           const Decide d = s_dec;
-          const ff x = ff_two_sum(d.zy, -mi);
-          const ff e = ff_exp_nonpos(x.hi, x.lo, s_th, s_tl);
-          const double ratio = ff_to_double(e) / (ff_to_double(zf) * (double)d.qy);
+          // p(y) / q(y) in double precision: z(y) - m is exact as a double, and neither p(y) nor a
+          // subnormal q(y) leaves the double range
+          const double ratio = exp((double)d.zy - (double)mi) / (ff_to_double(zf) * (double)d.qy);
           s_walk[0] = (double)d.u <= fmin(1.0, ratio) ? 0 : 1;
         }
         __syncthreads();

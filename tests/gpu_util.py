@@ -38,13 +38,18 @@ def subset_rows(batch, reqs):
     return np.concatenate([np.arange(qs[r], qs[r + 1]) for r in reqs])
 
 
-def pick_requests(batch, n=6, seed=0):
-    """A sample of requests for full-size attention parity: longest, shortest, k extremes, random."""
-    B = batch.B
-    kv = batch.context_lens.astype(np.int64) + batch.draft_lens
-    picks = {int(np.argmax(kv)), int(np.argmin(kv)), int(np.argmax(batch.draft_lens)), int(np.argmin(batch.draft_lens)),
-             B - 1, 0}
-    rng = np.random.default_rng(seed)
-    while len(picks) < min(B, n):
-        picks.add(int(rng.integers(B)))
-    return sorted(picks)
+def request_groups(batch, max_row_keys=2e8):
+    """Consecutive groups of requests whose oracle attention work (query rows x visible keys x
+    heads) stays under max_row_keys each, so that every oracle call is bounded."""
+    kv = batch.context_lens.astype(np.int64) + batch.draft_lens + 1
+    work = (batch.draft_lens.astype(np.int64) + 1) * kv * batch.Hq
+    groups, cur, acc = [], [], 0
+    for r in range(batch.B):
+        if cur and acc + work[r] > max_row_keys:
+            groups.append(cur)
+            cur, acc = [], 0
+        cur.append(r)
+        acc += int(work[r])
+    if cur:
+        groups.append(cur)
+    return groups

@@ -133,5 +133,6 @@ def test_empty_batch_is_a_no_op():
     wb.wisp_verify_attention(a, ws)
     wb.wisp_verify_accept(c, ws)
     torch.cuda.synchronize()
-    assert wb.wisp_verify_get_device_status(ws) == (0, 0)
+    # no error: code 0 and request id -1, as include/wisp_verify.h documents
+    assert wb.wisp_verify_get_device_status(ws) == (0, -1)
     assert out_L.item() == -7 and out_t.item() == -7
