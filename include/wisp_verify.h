@@ -180,7 +180,7 @@ wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args 
  * and allocates nothing.  No counterpart in the paper: it exists for callers that cannot allocate
  * device memory when they verify (memory owned by another allocator, or a latency path on which
  * cudaMalloc, which may synchronise the device, is not allowed).
- *   Scratch: a fixed 4 MiB array inside this library's device image, shared by every call in
+ *   Scratch: a fixed 16 MiB array inside this library's device image, shared by every call in
  *   the process.  Calls that overlap in time (other streams, other host threads) race on it and
  *   corrupt each other's results: order them, e.g. on one stream.
  *   Limit: B <= 8192 requests and total_q_rows <= 131072; a larger batch returns

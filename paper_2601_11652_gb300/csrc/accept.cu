@@ -1,47 +1,48 @@
 // accept.cu -- the in-order speculative acceptance pass over the vocabulary (Eq. 1-3).
 //
-// Two launches.
+// One persistent kernel, accept_kernel, with two kinds of work taken from device-side queues:
 //
-// row_stats_kernel: warp (row, slice) streams one vocabulary slice of one logit row once, as
-// 16-byte vectors; every lane keeps a running max, a double-float running sum of exp(z - max)
-// (fp32 terms, pairwise within a vector) and the terms of a certified bound on the relative
-// error of the normaliser Z (exp error, rounding of the argument, every rescale, pairwise sums);
-// the warp merges them into the slice's statistics.  Every row of the batch is processed, in
-// parallel, so the pass runs at HBM bandwidth; rows past a request's first rejection are read
-// although the rule never uses them.
+// Statistics items (row, slice), dispatched level-major (row index 0 of every request, then row
+// index 1, ...), so that by the time row i of a request comes up its earlier decisions are usually
+// known and rows past a rejection -- which the rule never reads -- are skipped.  A CTA streams its
+// slice once as 16-byte vectors; every thread keeps a running max, a double-float sum of
+// exp(z - m) (hardware 2^x) and the terms of a certified bound on the relative error of that sum.
+// The CTA that finishes the last slice of a row merges the slices and takes the decision the row
+// scores (Eq. 1, a = min(1, p(y)/q(y)), accept iff u <= a) in fp32 when u lies outside the
+// certified interval of the ratio, else after recomputing the row's normaliser exactly.  It then
+// checks whether the request's accepted length L is now known (Eq. 2: the first rejection, or k)
+// and, if so, queues the request for its draw.
 //
-// accept_kernel: one thread-block cluster of C CTAs (C = 1..8, chosen from the batch size) per
-// request.  Walk (Eq. 1-2): warp w merges the slice statistics of row i0 + w (rows in batches
-// of 8; row i scores draft token i+1, row k is the bonus row) and thread 0 takes the decisions
-// u_i <= min(1, p(y)/q(y)) in order, in fp32 when u_i lies outside the certified interval of the
-// ratio; otherwise the cluster recomputes that row's Z and p(y) in double-float arithmetic
-// (Tang's table-driven exp) and decides on those.  The walk stops at the first rejection.
-// Draw (Eq. 3): from max(0, p_L - q_{L+1}) after a rejection, else from p_L, by inverse CDF in
-// ascending token order: CTA c owns a contiguous slice of the row; one double-float sweep gives
-// per-(round, warp) tile sums in shared memory and per-CTA totals (through distributed shared
-// memory, summed in rank order so every CTA holds bit-identical values); the CTA holding the
-// crossing of u * total scans its tiles, then one warp scans the tile, then one lane its
-// elements.
+// Draw items (request, slice of row L) for the extra token (Eq. 3): the residual
+// max(0, p_L - q_{L+1}) after a rejection, else p_L, by inverse CDF in ascending token order.  The
+// weights exp(z - m) are exact 64-bit fixed-point numbers (a per-CTA table over the bf16 values,
+// computed in double-float), so every sum is exact and independent of its order.  One pass gives,
+// per slice, the sum over all elements (the exact normaliser) and, over the elements with
+// p > q, the sums of exp(z - m) and of q; the residual mass of a slice is then
+// E_P - Z Q_P once Z is known.  Elements whose sign the fp32 normaliser cannot settle are kept
+// aside and weighed exactly.  The CTA that finishes the last slice of a request finds the slice
+// holding the crossing of u * total, rescans it with the exact normaliser and writes the token.
+//
+// Nothing waits on an unbounded condition: a CTA that finds no work sleeps briefly and gives up
+// after about two seconds (recording WISP_DEV_TIMEOUT); the only other wait is for a queue entry
+// whose slot was already reserved by a running CTA.
 #include <cfloat>
-#include <cooperative_groups.h>
+#include <cmath>
 #include <cstring>
 #include <type_traits>
 
 #include "accept.cuh"
-
-namespace cg = cooperative_groups;
+#include "sm100_ptx.cuh"
 
 namespace wisp {
+
+// exp(u) for the bf16 values u of the draw's table (double-float), written by accept_setup
+__device__ ff g_exp_u[kExpTabSize];
 
 namespace {
 
 constexpr int NW = kAcceptThreads / 32;
 constexpr int NT = kAcceptThreads;
-// vectors (normaliser passes) and rounds (draw sweep) a thread keeps loaded ahead of the one it
-// uses, in a ring of registers with one copy of the loop body: with one 16-byte load in flight per
-// thread the streams of accept_kernel are latency-bound
-constexpr int kZAhead = 8;
-constexpr int kSweepAhead = 4;
 
 template <typename LT>
 struct LTraits;
@@ -113,9 +114,12 @@ __device__ __forceinline__ void load_q(const float *qrow, int64_t v0, int V, boo
   }
 }
 
-// bf16 logits take few distinct values, so the draw looks exp(u - m) up in a table of the bf16
-// values u in the table's range, computed once per CTA with the very same double-float function
-// (the results are bit-identical to computing every element); other values are computed directly.
+// Accesses to the launch's shared state (other CTAs write it; L1 is not coherent).
+__device__ __forceinline__ int ld_vol(const int32_t *p) { return *(const volatile int32_t *)p; }
+__device__ __forceinline__ void st_vol(int32_t *p, int v) { *(volatile int32_t *)p = v; }
+__device__ __forceinline__ void fence_sc() { asm volatile("fence.sc.gpu;" ::: "memory"); }
+
+// ---- the draw's exp table --------------------------------------------------------------------
 __device__ __forceinline__ int exp_tab_index(uint32_t bits16) {
   const uint32_t d = ((bits16 >> 7) & 0xFFu) - (uint32_t)kExpTabLo;  // wraps below the range
   if (d >= (uint32_t)kExpTabBinades) return -1;
@@ -126,77 +130,107 @@ __device__ __forceinline__ uint32_t exp_tab_bits(int idx) {
   return (sign << 15) | (((rem >> 7) + kExpTabLo) << 7) | (rem & 0x7Fu);
 }
 
-// Double-float weight of one element in the draw: exp(z - m) [- q * Z, clamped at 0].
-__device__ __forceinline__ ff draw_weight(float z, float m, bool residual, float q, ff Zff, const float *th,
-                                          const float *tl) {
+// round(2^56 x) for |x| <= 1 from the bits of x (integer operations only: 64-bit conversions run
+// on the slow FP64 pipe); zero below 2^-126.
+__device__ __forceinline__ long long f32_to_fix(float x) {
+  const uint32_t b = __float_as_uint(x);
+  const int e = (int)((b >> 23) & 0xFFu);
+  if (e == 0) return 0;
+  const unsigned long long mant = (unsigned long long)((b & 0x7FFFFFu) | 0x800000u);  // x = mant 2^(e - 150)
+  const int sh = e - 150 + kFixShift;
+  unsigned long long v;
+  if (sh >= 0)
+    v = mant << sh;
+  else if (sh > -40)
+    v = (mant + (1ull << (-sh - 1))) >> (-sh);
+  else
+    v = 0;
+  return (b >> 31) ? -(long long)v : (long long)v;
+}
+// round(2^56 a) for a double-float a in [0, 1] (the two parts converted exactly up to the last
+// half unit and added).
+__device__ __forceinline__ unsigned long long ff_to_fix(ff a) {
+  const long long r = f32_to_fix(a.hi) + f32_to_fix(a.lo);
+  return r > 0 ? (unsigned long long)r : 0ull;
+}
+
+// A draw weight: round(2^56 exp(z - m)) and exp(z - m) rounded to float.
+struct Wt {
+  unsigned long long fix;
+  float f;
+};
+
+// exp(z - m), z <= m, computed directly (double-float, Tang's method).
+__device__ __noinline__ Wt exp_fix_direct(float z, float m, const float *th, const float *tl) {
   const ff x = ff_two_sum(z, -m);
-  ff e = ff_exp_nonpos(x.hi, x.lo, th, tl);
-  if (residual) {
-    e = ff_add(e, ff_neg(ff_mul_f(Zff, q)));
-    if (!(e.hi > 0.0f)) e = {0.0f, 0.0f};
-  }
-  return e;
+  const ff e = ff_exp_nonpos(x.hi, x.lo, th, tl);
+  return Wt{ff_to_fix(e), e.hi};
 }
 
-// Out-of-table values (rare for logits): the direct double-float exp, kept out of line so that the
-// unrolled loops stay small.
-__device__ __noinline__ ff exp_direct(float z, float m, const float *th, const float *tl) {
-  return draw_weight(z, m, false, 0.0f, ff{}, th, tl);
+// s += q exactly as a double-float without renormalisation (Knuth's TwoSum; the low part collects
+// the rounding errors).
+__device__ __forceinline__ void ff_acc(ff &s, float q) {
+  const float t = __fadd_rn(s.hi, q);
+  const float bp = __fsub_rn(t, s.hi);
+  const float ap = __fsub_rn(t, bp);
+  s.lo = __fadd_rn(s.lo, __fadd_rn(__fsub_rn(s.hi, ap), __fsub_rn(q, bp)));
+  s.hi = t;
 }
 
-// exp(z - m) of element i of vector w; bf16: from the table when z is in its range.
-template <typename LT>
-__device__ __forceinline__ ff elem_exp(const uint4 &w, int i, float m, const ff *tab, const float *th, const float *tl);
-template <>
-__device__ __forceinline__ ff elem_exp<float>(const uint4 &w, int i, float m, const ff *, const float *th, const float *tl) {
-  return draw_weight(vec_elem<float>(w, i), m, false, 0.0f, ff{}, th, tl);
+__device__ __forceinline__ void u96_add(U96 &a, unsigned long long x) {
+  const unsigned long long o = a.lo;
+  a.lo += x;
+  a.hi += (a.lo < o) ? 1u : 0u;
 }
-template <>
-__device__ __forceinline__ ff elem_exp<uint16_t>(const uint4 &w, int i, float m, const ff *tab, const float *th,
-                                                 const float *tl) {
-  const uint32_t u = (i >> 1) == 0 ? w.x : (i >> 1) == 1 ? w.y : (i >> 1) == 2 ? w.z : w.w;
-  const int idx = exp_tab_index((i & 1) ? (u >> 16) : (u & 0xFFFFu));
-  if (tab && idx >= 0) return tab[idx];
-  return exp_direct(vec_elem<uint16_t>(w, i), m, th, tl);
+__device__ __forceinline__ void u96_add(U96 &a, const U96 &b) {
+  u96_add(a, b.lo);
+  a.hi += b.hi;
 }
-
-// Sum of two non-negative double-float values: Dekker's addition without the TwoSum of the low
-// parts.  With operands of one sign no cancellation occurs and the relative error stays within
-// about 3 * 2^-48 (the full ff_add is kept wherever a difference is formed).
-__device__ __forceinline__ ff ff_add_pos(ff a, ff b) {
-  ff s = ff_two_sum(a.hi, b.hi);
-  s.lo = __fadd_rn(s.lo, __fadd_rn(a.lo, b.lo));
-  return ff_fast_two_sum(s.hi, s.lo);
+__device__ __forceinline__ double u96_to_double(const U96 &a) { return (double)a.hi * 0x1p64 + (double)a.lo; }
+__device__ __forceinline__ U96 u96_zero() {
+  U96 r;
+  r.lo = 0;
+  r.hi = 0;
+  r.pad = 0;
+  return r;
 }
-
-// Pairwise sum of the E non-negative terms of one vector (three levels for E = 8).
-template <int E>
-__device__ __forceinline__ ff ff_tree_pos(ff (&t)[E]) {
-#pragma unroll
-  for (int w = 1; w < E; w <<= 1) {
-#pragma unroll
-    for (int i = 0; i < E; i += 2 * w) t[i] = ff_add_pos(t[i], t[i + w]);
-  }
-  return t[0];
+__device__ __forceinline__ U96 u96_shfl_xor(const U96 &a, int o) {
+  U96 r;
+  r.lo = __shfl_xor_sync(0xffffffffu, a.lo, o);
+  r.hi = __shfl_xor_sync(0xffffffffu, a.hi, o);
+  r.pad = 0;
+  return r;
+}
+__device__ __forceinline__ U96 u96_warp_sum(U96 a) {
+  for (int o = 16; o > 0; o >>= 1) u96_add(a, u96_shfl_xor(a, o));
+  return a;
 }
 
-// Draw weight from e = exp(z - m): e itself, or the residual max(0, e - q Z) (as draw_weight).
-__device__ __forceinline__ ff weight_from(ff e, bool residual, float q, ff Zff) {
-  if (residual) {
-    e = ff_add(e, ff_neg(ff_mul_f(Zff, q)));
-    if (!(e.hi > 0.0f)) e = {0.0f, 0.0f};
-  }
-  return e;
+}  // namespace
+
+namespace {
+
+// ---- row statistics (Eq. 1 needs p = softmax of the row) ----------------------------------------
+__device__ __forceinline__ uint32_t bmax2_nan(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("max.NaN.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+__device__ __forceinline__ float fmax_nan(float a, float b) {
+  float r;
+  asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+  return r;
 }
 
-
-// Per-thread streaming statistics of one row slice (see the file comment).
+// Per-thread streaming statistics of a row slice: running max m, double-float sum s of
+// exp(z - m), A = sum exp(z - m) |z - m| (bounds the effect of rounding z - m and its product with
+// log2 e), rescales so far, and the first finite max (bounds the size of all rescale arguments).
 struct RowStats {
-  float m;       // running max
-  ff s;          // sum of exp(z - m)
-  float A;       // sum of exp(z - m) * |z - m|  (bounds the effect of rounding z - m)
-  int nres;      // rescales so far
-  float mfirst;  // first finite max (bounds the size of all rescale arguments)
+  float m;
+  ff s;
+  float A;
+  int nres;
+  float mfirst;
 };
 
 __device__ __forceinline__ void stats_init(RowStats &st) {
@@ -207,9 +241,13 @@ __device__ __forceinline__ void stats_init(RowStats &st) {
   st.mfirst = INFINITY;
 }
 
-// Move the statistics to a larger reference max mnew.
+// Move the statistics to a larger reference max mnew (NaN propagates into m).
 __device__ __forceinline__ void stats_rebase(RowStats &st, float mnew) {
   if (st.m == -INFINITY) {
+    st.m = mnew;
+    return;
+  }
+  if (mnew != mnew) {
     st.m = mnew;
     return;
   }
@@ -222,75 +260,107 @@ __device__ __forceinline__ void stats_rebase(RowStats &st, float mnew) {
   st.nres += 1;
 }
 
-// Add one chunk of NV vectors (a thread's next elements of its slice): the chunk max first (one
-// rescale at most per chunk), then exp(z - m) = 2^((z - m) * log2 e) per element, a pairwise fp32
-// sum of the chunk added to the double-float running sum, and the bound term A.
+// Max of the chunk's elements (NaN if any is NaN): bf16 pairs two at a time, then the two halves.
+template <typename LT, int NV>
+__device__ __forceinline__ float chunk_max(const uint4 (&w)[NV]) {
+  if (std::is_same<LT, uint16_t>::value) {
+    uint32_t a = bmax2_nan(w[0].x, w[0].y), b = bmax2_nan(w[0].z, w[0].w);
+#pragma unroll
+    for (int u = 1; u < NV; ++u) {
+      a = bmax2_nan(a, bmax2_nan(w[u].x, w[u].y));
+      b = bmax2_nan(b, bmax2_nan(w[u].z, w[u].w));
+    }
+    a = bmax2_nan(a, b);
+    return fmax_nan(__uint_as_float(a << 16), __uint_as_float(a & 0xffff0000u));
+  }
+  float a = fmax_nan(__uint_as_float(w[0].x), __uint_as_float(w[0].y));
+  float b = fmax_nan(__uint_as_float(w[0].z), __uint_as_float(w[0].w));
+#pragma unroll
+  for (int u = 1; u < NV; ++u) {
+    a = fmax_nan(a, fmax_nan(__uint_as_float(w[u].x), __uint_as_float(w[u].y)));
+    b = fmax_nan(b, fmax_nan(__uint_as_float(w[u].z), __uint_as_float(w[u].w)));
+  }
+  return fmax_nan(a, b);
+}
+
+// Min of the chunk's elements (NaN ignored: a NaN already makes the max NaN).
+template <typename LT, int NV>
+__device__ __forceinline__ float chunk_min(const uint4 (&w)[NV]) {
+  if (std::is_same<LT, uint16_t>::value) {
+    uint32_t a, b;
+    asm("min.bf16x2 %0, %1, %2;" : "=r"(a) : "r"(w[0].x), "r"(w[0].y));
+    asm("min.bf16x2 %0, %1, %2;" : "=r"(b) : "r"(w[0].z), "r"(w[0].w));
+#pragma unroll
+    for (int u = 1; u < NV; ++u) {
+      uint32_t c, d;
+      asm("min.bf16x2 %0, %1, %2;" : "=r"(c) : "r"(w[u].x), "r"(w[u].y));
+      asm("min.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(w[u].z), "r"(w[u].w));
+      asm("min.bf16x2 %0, %1, %2;" : "=r"(a) : "r"(a), "r"(c));
+      asm("min.bf16x2 %0, %1, %2;" : "=r"(b) : "r"(b), "r"(d));
+    }
+    asm("min.bf16x2 %0, %1, %2;" : "=r"(a) : "r"(a), "r"(b));
+    return fminf(__uint_as_float(a << 16), __uint_as_float(a & 0xffff0000u));
+  }
+  float a = fminf(__uint_as_float(w[0].x), __uint_as_float(w[0].y));
+  float b = fminf(__uint_as_float(w[0].z), __uint_as_float(w[0].w));
+#pragma unroll
+  for (int u = 1; u < NV; ++u) {
+    a = fminf(a, fminf(__uint_as_float(w[u].x), __uint_as_float(w[u].y)));
+    b = fminf(b, fminf(__uint_as_float(w[u].z), __uint_as_float(w[u].w)));
+  }
+  return fminf(a, b);
+}
+
+// Add one chunk of vectors: its max first (one rescale at most per chunk), then
+// exp(z - m) = 2^((z - m) log2 e) per element, a pairwise fp32 sum of the chunk (vector trees, then
+// across the vectors) added to the double-float running sum, and the bound term A, here
+// (chunk sum) * min(m - chunk min, 104) >= sum exp(z - m) |z - m| (below 104 every term is < 2^-150).
 template <typename LT, int NV>
 __device__ __forceinline__ void stats_add_chunk(RowStats &st, const uint4 (&w)[NV]) {
   constexpr int E = LTraits<LT>::E;
-  constexpr int N = NV * E;
-  float z[N];
-#pragma unroll
-  for (int u = 0; u < NV; ++u) {
-#pragma unroll
-    for (int i = 0; i < E; ++i) z[u * E + i] = vec_elem<LT>(w[u], i);
-  }
-  float mx[8];
-#pragma unroll
-  for (int i = 0; i < 8; ++i) mx[i] = z[i];
-#pragma unroll
-  for (int i = 8; i < N; ++i) mx[i & 7] = fmaxf(mx[i & 7], z[i]);
-  const float cm = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+  const float cm = chunk_max<LT, NV>(w);
   if (cm == -INFINITY) return;  // nothing but padding (or -inf logits)
   if (st.m == -INFINITY) st.mfirst = cm;
   stats_rebase(st, cm);
-  float e[N];
-  float a[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+  const float m = st.m;
+  const float span = fminf(m - chunk_min<LT, NV>(w), 104.0f);
+  float vs[NV];
 #pragma unroll
-  for (int i = 0; i < N; ++i) {
-    const float x = z[i] - st.m;
-    e[i] = ex2_approx(x * kLog2e);
-    a[i & 3] = fmaf(e[i], fminf(-x, 104.0f), a[i & 3]);
+  for (int u = 0; u < NV; ++u) {
+    float e[E];
+#pragma unroll
+    for (int i = 0; i < E; ++i) {
+      const float x = vec_elem<LT>(w[u], i) - m;
+      e[i] = ex2_approx(x * kLog2e);
+    }
+#pragma unroll
+    for (int h = 1; h < E; h <<= 1) {
+#pragma unroll
+      for (int i = 0; i < E; i += 2 * h) e[i] += e[i + h];
+    }
+    vs[u] = e[0];
   }
 #pragma unroll
-  for (int w2 = 1; w2 < N; w2 <<= 1) {
+  for (int h = 1; h < NV; h <<= 1) {
 #pragma unroll
-    for (int i = 0; i < N; i += 2 * w2) e[i] += e[i + w2];
+    for (int u = 0; u + h < NV; u += 2 * h) vs[u] += vs[u + h];
   }
-  st.s = ff_add_f(st.s, e[0]);
-  st.A += (a[0] + a[1]) + (a[2] + a[3]);
+  st.s = ff_add_f(st.s, vs[0]);
+  st.A = fmaf(vs[0], span, st.A);
 }
 
-struct Decide {
-  int flag;  // 0 accept, 1 reject, 2 uncertain, 4 bad prob
-  float zy, qy, u;
-};
-
-// Warp-wide merge of the S <= 32 slice statistics of one row (lane q reads slice q): the same
-// max / rebase / tree-sum, so every lane (and every CTA that does it) holds identical values.
-// The slice-to-row rebase is not counted in nres; the decision bound allows for it.
-__device__ __forceinline__ RowStats merge_parts(const RowPart *parts, int S) {
-  const int lane = threadIdx.x & 31;
-  RowStats q;
-  stats_init(q);
-  if (lane < S) {
-    const RowPart t = parts[lane];
-    q.m = t.m;
-    q.s = {t.s_hi, t.s_lo};
-    q.A = t.A;
-    q.mfirst = t.mfirst;
-    q.nres = t.nres;
-  }
-  float gm = q.m, gf = q.mfirst;
-  int gn = q.nres;
+// Warp-wide merge of per-lane statistics: max, rebase, tree sum (every lane ends with the result).
+__device__ __forceinline__ RowStats warp_merge(RowStats st) {
+  float gm = st.m, gf = st.mfirst;
+  int gn = st.nres;
   for (int o = 16; o > 0; o >>= 1) {
-    gm = fmaxf(gm, __shfl_xor_sync(0xffffffffu, gm, o));
+    gm = fmax_nan(gm, __shfl_xor_sync(0xffffffffu, gm, o));
     gf = fminf(gf, __shfl_xor_sync(0xffffffffu, gf, o));
     gn = max(gn, __shfl_xor_sync(0xffffffffu, gn, o));
   }
-  if (q.m > -INFINITY) stats_rebase(q, gm);
-  ff gs = q.m > -INFINITY ? q.s : ff{0.0f, 0.0f};
-  float ga = q.m > -INFINITY ? q.A : 0.0f;
+  if (st.m > -INFINITY) stats_rebase(st, gm);
+  ff gs = st.m > -INFINITY ? st.s : ff{0.0f, 0.0f};
+  float ga = st.m > -INFINITY ? st.A : 0.0f;
   for (int o = 16; o > 0; o >>= 1) {
     gs = ff_add(gs, ff_shfl_xor(gs, o));
     ga += __shfl_xor_sync(0xffffffffu, ga, o);
@@ -299,513 +369,1250 @@ __device__ __forceinline__ RowStats merge_parts(const RowPart *parts, int S) {
   r.m = gm;
   r.s = gs;
   r.A = ga;
-  r.nres = gn;
+  r.nres = gn + 1;  // the lane-to-warp rebase
   r.mfirst = gf;
   return r;
 }
 
+// Certified relative error of a row's normaliser Z~ (see RowStats): one 2^x error per element and
+// per rescale on its way (thread, warp, CTA, row), three roundings in the argument of every element
+// and every rescale, the pairwise fp32 sums; the double-float additions are covered by 1e-12.
+__device__ __forceinline__ float z_bound(const RowStats &rs) {
+  return 1.05f * ((float)(rs.nres + 2) * kEx2RelErr + 3.0f * 0x1p-24f * (rs.m - rs.mfirst) +
+                  3.0f * 0x1p-24f * (rs.A / rs.s.hi) + 6.0f * 0x1p-24f) +
+         1e-12f;
+}
+
 }  // namespace
 
-// Statistics of one vocabulary slice of one logit row (Eq. 1 needs p = softmax of the row):
-// warp (row, slice) streams its slice once, every lane keeping a running max, a double-float sum
-// of exp(z - m) and the error terms over chunks of 4 vectors (the next chunk's loads are issued
-// before the current one is reduced); the lanes are merged with shuffles (max, rebase, tree sum)
-// and lane 0 writes the slice's statistics.  No shared memory, no block barrier.
-template <typename LT>
-__global__ void __launch_bounds__(NT) row_stats_kernel(const __grid_constant__ AcceptParams p) {
-  constexpr int E = LTraits<LT>::E;
-  const int lane = threadIdx.x & 31;
-  const int64_t unit = (int64_t)blockIdx.x * NW + (threadIdx.x >> 5);
-  if (unit >= p.total_rows * p.slices) return;
-  const int64_t row = unit / p.slices;
-  const int sl = (int)(unit % p.slices);
-  const int V = p.V;
-  const LT *rowp = static_cast<const LT *>(p.logits) + row * (int64_t)V;
-  const bool vec_z = p.vec_z != 0;
-  const int64_t nvec = (V + E - 1) / E;
-  const int64_t vlo = min(nvec, (int64_t)sl * p.vps);
-  const int64_t vhi = min(nvec, vlo + p.vps);
-  const uint32_t ni = LTraits<LT>::NEG_INF2;
-  auto load4 = [&](int64_t base, uint4 (&w)[4]) {
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int64_t vi = base + u * 32;
-      w[u] = vi < vhi ? load_vec<LT>(rowp, vi, V, vec_z) : make_uint4(ni, ni, ni, ni);
+namespace {
+
+// ---- the persistent acceptance kernel: roles, items, shared state ----------------------------
+// Warps 0..7 consume (compute from shared memory), warp 8 produces (picks the next item and keeps
+// bulk copies of its rows in flight in a ring of stages), warp 9 keeps the books (slice records,
+// atomics, the row decisions, L, the draw's crossing search).
+enum : int { WORK_EXIT = 0, WORK_WAIT = 1, WORK_STATS = 2, WORK_DRAW = 3, WORK_FINISH = 4 };
+enum : int { ROW_UNCERTAIN = 100 };  // transient: decided by the exact normaliser
+
+constexpr int kConsumers = kAcceptThreads;    // consumer threads
+constexpr int kCW = kConsumers / 32;          // consumer warps
+constexpr int kProducerWarp = kCW;
+constexpr int kCtaThreads = kConsumers + 64;
+constexpr int kStages = 5;
+constexpr int kStageBytes = 12288;
+constexpr int kStatsChunk = kConsumers * kStatsChunkVecs;  // vectors per statistics chunk (12 KB)
+constexpr int kDrawChunk = kConsumers;        // vectors per draw chunk: z 4 KB + q up to 8 KB
+constexpr int kDrawTile = kDrawChunk / (kCW / 2);  // vectors per tile: one warp's share of a draw chunk
+constexpr int kQOffset = 4096;                // the q part of a draw chunk within its stage
+constexpr int kItemSlots = 4;
+constexpr int kFinQ = 8;
+constexpr long long kWaitCycles = 4000000000LL;  // about two seconds: a wait that long is a failure
+constexpr size_t kRingBytes = (size_t)kStages * kStageBytes;
+static_assert(kDrawChunk * 16 <= kQOffset && kQOffset + kDrawChunk * 8 * 4 <= kStageBytes, "draw chunk layout");
+static_assert(kStatsChunk * 16 <= kStageBytes, "statistics chunk layout");
+
+// One unit of work, written by the producer into an item slot, read by the consumers and the keeper.
+struct Item {
+  int kind, r, i, s, k, resid;
+  int64_t R, Q0, D0;
+  int64_t v0, v1;  // vectors [v0, v1) of the row streamed
+  int nchunks;
+  RowRec rec;
+  // finish: the vectors holding the crossing ([v0, v1)) and its local threshold
+  double thr, Zu;
+  int take_last;
+  // results of the consumers
+  SlicePart sp;
+  U96 ea, ep;
+  ff qp;
+  int n_amb;
+  AmbElem amb[kAmbPerSlice];
+};
+
+// A draw to finish on this CTA (posted by the keeper, scheduled by the producer).
+struct FinTask {
+  int r, i, k, resid, take_last;
+  int64_t Q0, D0, v0, v1;  // the vectors to search: one tile, or a whole slice
+  RowRec rec;
+  double thr, Zu;
+};
+
+// The draw's per-CTA exp table (dynamic shared memory): the fixed-point value as two 32-bit words
+// and the float value, three arrays of 4-byte entries (random 4-byte loads cost far less than
+// random 8-byte ones).
+struct Tab {
+  uint32_t *lo, *hi;
+  float *f;
+};
+
+struct Sm {
+  uint64_t full[kStages], empty[kStages];
+  uint64_t iq_full[kItemSlots], iq_empty[kItemSlots], res_ready[kItemSlots];
+  uint64_t cons_bar;  // the consumers' barrier (an mbarrier, so that every wait is bounded)
+  Item item[kItemSlots];
+  float th[256], tl[256];  // 2^(j/256) as double-float pairs (Tang's exp)
+  // consumers
+  RowStats wst[kCW];
+  U96 red[2][2][kCW];  // [buffer][e_all, e_p][warp]
+  ff qred[2][kCW];
+  double dred[kCW];
+  unsigned tab_m_bits;
+  int tab_valid;
+  int amb_n;
+  AmbElem amb[kAmbPerSlice];
+  int first, lastpos;
+  // local finish queue (keeper -> producer)
+  FinTask fq[kFinQ];
+  int fq_head, fq_tail;
+  int keeper_done;
+  int abort_;
+};
+
+__device__ __forceinline__ int vload(const int &x) { return *(const volatile int *)&x; }
+__device__ __forceinline__ void vstore(int &x, int v) { *(volatile int *)&x = v; }
+
+// Bounded wait for the phase of `bar` with parity `parity`; false after about two seconds or once
+// another role gave up (every role then leaves its loop).
+__device__ bool wait_bar(uint64_t *bar, uint32_t parity, Sm &sm, const AcceptParams &p) {
+  if (ptx::mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  // suspended in the barrier between the checks, so that waiting warps leave the issue slots to
+  // the ones that compute
+  while (!ptx::mbar_try_wait_sleep(bar, parity, 20000)) {
+    if (vload(sm.abort_)) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      if (atomicExch(&sm.abort_, 1) == 0) report(p.status, WISP_DEV_TIMEOUT, nullptr, -1);
+      return false;
     }
-  };
-  RowStats st;
-  stats_init(st);
-  uint4 cur[4];
-  load4(vlo + lane, cur);
-  for (int64_t base = vlo + lane; base < vhi; base += 4 * 32) {
-    uint4 nxt[4];
-    load4(base + 4 * 32, nxt);
-    stats_add_chunk<LT, 4>(st, cur);
+  }
+  return true;
+}
+
+// Barrier of the consumer threads: every consumer arrives, then waits (bounded) for the phase;
+// `ph` counts this thread's barriers.
+__device__ __forceinline__ void cbar(Sm &sm, uint32_t &ph, const AcceptParams &p) {
+  ptx::mbar_arrive(&sm.cons_bar);
+  wait_bar(&sm.cons_bar, ph & 1, sm, p);
+  ++ph;
+}
+
+// Build the per-CTA table of round(2^56 exp(u - m)) over the table's bf16 values u (0 for u > m),
+// unless it already holds this m: from exp(u) exp(-m) when -m is itself a table value, else
+// directly; both in double-float.  Called by every consumer thread.
+__device__ void ensure_table(float m, Sm &sm, Tab tab, uint32_t &ph, const AcceptParams &p) {
+  constexpr int PER = (kExpTabSize + kConsumers - 1) / kConsumers;
+  const unsigned mb = __float_as_uint(m);
+  if (sm.tab_valid && sm.tab_m_bits == mb) return;
+  cbar(sm, ph, p);  // no consumer still reads the previous table
+  const int mi = exp_tab_index((mb >> 16) ^ 0x8000u);  // -m (m is a bf16 value)
+  if (mi >= 0) {
+    const ff Em = g_exp_u[mi];
+    ff g[PER];  // every load first: one round trip
 #pragma unroll
-    for (int u = 0; u < 4; ++u) cur[u] = nxt[u];
+    for (int j = 0; j < PER; ++j) {
+      const int idx = threadIdx.x + j * kConsumers;
+      g[j] = idx < kExpTabSize ? g_exp_u[idx] : ff{0.0f, 0.0f};
+    }
+#pragma unroll
+    for (int j = 0; j < PER; ++j) {
+      const int idx = threadIdx.x + j * kConsumers;
+      if (idx < kExpTabSize) {
+        const bool used = bf16_bits_to_float(exp_tab_bits(idx)) <= m;
+        const ff e = ff_mul(g[j], Em);
+        const unsigned long long fx = used ? ff_to_fix(e) : 0ull;
+        tab.lo[idx] = (uint32_t)fx;
+        tab.hi[idx] = (uint32_t)(fx >> 32);
+        tab.f[idx] = used ? e.hi : 0.0f;
+      }
+    }
+  } else {
+    for (int idx = threadIdx.x; idx < kExpTabSize; idx += kConsumers) {
+      const float u = bf16_bits_to_float(exp_tab_bits(idx));
+      const Wt v = u <= m ? exp_fix_direct(u, m, sm.th, sm.tl) : Wt{0, 0.0f};
+      tab.lo[idx] = (uint32_t)v.fix;
+      tab.hi[idx] = (uint32_t)(v.fix >> 32);
+      tab.f[idx] = v.f;
+    }
   }
-  // lanes -> slice: max, rebase, tree sum (the lane-to-slice rebase counts as one more rescale)
-  float wm = st.m, wf = st.mfirst;
-  int wn = st.nres;
-  for (int o = 16; o > 0; o >>= 1) {
-    wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
-    wf = fminf(wf, __shfl_xor_sync(0xffffffffu, wf, o));
-    wn = max(wn, __shfl_xor_sync(0xffffffffu, wn, o));
+  if (threadIdx.x == 0) {
+    sm.tab_m_bits = mb;
+    sm.tab_valid = 1;
   }
-  if (wm > -INFINITY) stats_rebase(st, wm);
-  ff ws = st.m > -INFINITY ? st.s : ff{0.0f, 0.0f};
-  float wa = st.m > -INFINITY ? st.A : 0.0f;
-  for (int o = 16; o > 0; o >>= 1) {
-    ws = ff_add(ws, ff_shfl_xor(ws, o));
-    wa += __shfl_xor_sync(0xffffffffu, wa, o);
+  cbar(sm, ph, p);
+}
+
+// The E weights of one vector: round(2^56 exp(z - m)) and exp(z - m) as a float.  From the table for
+// bf16 values in its range (almost every logit); the others (|z| < 2^-8, |z| >= 64, +-0, a table
+// not given) directly, entered once per vector that needs it.
+template <typename LT>
+__device__ __forceinline__ void weights(const uint4 &w, float m, const Sm &sm, Tab tab,
+                                        unsigned long long (&fx)[LTraits<LT>::E], float (&fl)[LTraits<LT>::E]);
+template <>
+__device__ __forceinline__ void weights<uint16_t>(const uint4 &w, float m, const Sm &sm, Tab tab,
+                                                  unsigned long long (&fx)[8], float (&fl)[8]) {
+  bool slow = false;
+  int idx[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const uint32_t u = (i >> 1) == 0 ? w.x : (i >> 1) == 1 ? w.y : (i >> 1) == 2 ? w.z : w.w;
+    const uint32_t bits = (i & 1) ? (u >> 16) : (u & 0xFFFFu);
+    idx[i] = tab.lo ? exp_tab_index(bits) : -1;
+    if (bits == 0xFF80u) idx[i] = -2;  // -inf: a masked token
+    slow |= idx[i] == -1;
   }
-  if (lane == 0) {
-    RowPart out;
-    out.m = wm;
-    out.s_hi = ws.hi;
-    out.s_lo = ws.lo;
-    out.A = wa;
-    out.mfirst = wf;
-    out.nres = wn + 1;
-    p.parts[unit] = out;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    fx[i] = idx[i] >= 0 ? ((unsigned long long)tab.hi[idx[i]] << 32) | tab.lo[idx[i]] : 0ull;
+    fl[i] = idx[i] >= 0 ? tab.f[idx[i]] : 0.0f;
+  }
+  if (slow) {
+    #pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      if (idx[i] == -1) {
+        const Wt e = exp_fix_direct(vec_elem<uint16_t>(w, i), m, sm.th, sm.tl);
+        fx[i] = e.fix;
+        fl[i] = e.f;
+      }
+    }
+  }
+}
+template <>
+__device__ __forceinline__ void weights<float>(const uint4 &w, float m, const Sm &sm, Tab,
+                                               unsigned long long (&fx)[4], float (&fl)[4]) {
+  #pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const Wt e = exp_fix_direct(vec_elem<float>(w, i), m, sm.th, sm.tl);
+    fx[i] = e.fix;
+    fl[i] = e.f;
   }
 }
 
+__device__ __forceinline__ double ff_to_double_(ff a) { return (double)a.hi + (double)a.lo; }
+__device__ __forceinline__ ff ff_warp_sum(ff a) {
+  for (int o = 16; o > 0; o >>= 1) a = ff_add(a, ff_shfl_xor(a, o));
+  return a;
+}
+
+// Draw weight of one element in units of 2^-56, in double: the residual max(0, e - q Z) (Z = Zu in
+// the same units) or e itself.  fmax drops a NaN q (no mass), as max(0, p - q) does.
+__device__ __forceinline__ double weight_d(unsigned long long e, float q, bool residual, double Zu) {
+  return residual ? fmax(0.0, (double)e - (double)q * Zu) : (double)e;
+}
+
+// Exact draw weight (units 2^-56, double) of one vector once the normaliser Zu is known: the sign of
+// p - q by an fp32 test with a 2^-20 margin, else in double.
 template <typename LT>
-__global__ void __launch_bounds__(NT, 2) accept_kernel(const __grid_constant__ AcceptParams p) {
+__device__ __forceinline__ double vec_weight(const uint4 &w, const float *q, bool residual, float m, double Zu,
+                                             const Sm &sm, Tab tab) {
   constexpr int E = LTraits<LT>::E;
-  extern __shared__ ff s_tile[];  // [rounds * NW] per-(round, warp) draw sums, then the exp table (bf16)
-  __shared__ float s_th[256], s_tl[256];
-  __shared__ RowStats s_wst[NW];
-  __shared__ RowStats s_pub[2];   // this CTA's published totals (ring of 2)
-  __shared__ ff s_tot[kMaxAcceptCluster];
-  __shared__ RowStats s_rows[NW]; // merged statistics of the rows being walked
-  __shared__ int s_walk[2];       // walk state, row within the batch
-  __shared__ float s_zy[kPreload], s_qy[kPreload], s_u[kPreload];
-  __shared__ Decide s_dec;
-  __shared__ int s_bad;
-  __shared__ int s_owner, s_take_last;
-  __shared__ ff s_thr;
+  unsigned long long fx[E];
+  float fl[E];
+  weights<LT>(w, m, sm, tab, fx, fl);
+  const float Zf = (float)(Zu * 0x1p-56);
+  const float zh = Zf * (1.0f + 0x1p-20f), zl = Zf * (1.0f - 0x1p-20f);
+  unsigned long long sp = 0;
+  ff sq = {0.0f, 0.0f};
+  double ad = 0.0;
+#pragma unroll
+  for (int i = 0; i < E; ++i) {
+    if (!residual) {
+      sp += fx[i];
+    } else if (q[i] >= 0.0f && fl[i] > q[i] * zh) {
+      sp += fx[i];
+      ff_acc(sq, q[i]);
+    } else if (fl[i] > q[i] * zl) {
+      ad += weight_d(fx[i], q[i], true, Zu);
+    }
+  }
+  return (double)sp - (residual ? Zu * ff_to_double_(sq) : 0.0) + ad;
+}
 
-  // launched as a programmatic dependent of the kernel before it: nothing is read before that
-  // grid has completed and its writes are visible
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  cg::cluster_group cluster = cg::this_cluster();
-  const int C = p.cluster;
-  const int rank = (int)cluster.block_rank();
-  const int r = blockIdx.x / C;
+}  // namespace
+
+namespace {
+
+// ---- consumers ----------------------------------------------------------------------------------
+// Statistics item: the slice's chunks from the ring (three vectors per thread; a stage is released
+// as soon as it is in registers), per-thread streaming statistics, merged into it.sp.
+template <typename LT>
+__device__ void c_stats(Sm &sm, Item &it, const char *ring, int &c, uint32_t &ph, const AcceptParams &p) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (r >= p.B) return;                 // whole clusters only (grid = B * C)
-  if (p.req_flag[r] != REQ_OK) return;  // uniform across the cluster
-
-  const int V = p.V;
-  const int k = p.draft_lens[r];
-  const int64_t Q0 = p.q_row_start[r], D0 = p.draft_start[r];
-  const LT *logits = static_cast<const LT *>(p.logits);
-  const bool vec_z = p.vec_z != 0, vec_q = p.vec_q != 0;
-  const int64_t nvec = (V + E - 1) / E;
-  const int64_t vlo = min((int64_t)nvec, (int64_t)rank * p.vpc);
-  const int64_t vhi = min((int64_t)nvec, vlo + p.vpc);
-  const int rounds = (int)((vhi - vlo + NT - 1) / NT);
-  int xslot = 0;
-
-  for (int i = tid; i < 256; i += NT) {
-    s_th[i] = p.tab.hi[i];
-    s_tl[i] = p.tab.lo[i];
+  const uint32_t ni = LTraits<LT>::NEG_INF2;
+  RowStats st;
+  stats_init(st);
+  for (int j = 0; j < it.nchunks; ++j) {
+    const int stg = c % kStages;
+    if (!wait_bar(&sm.full[stg], (c / kStages) & 1, sm, p)) return;
+    const uint4 *src = reinterpret_cast<const uint4 *>(ring + (size_t)stg * kStageBytes);
+    const int64_t nv = min((int64_t)kStatsChunk, it.v1 - (it.v0 + (int64_t)j * kStatsChunk));
+    uint4 w[kStatsChunkVecs];
+#pragma unroll
+    for (int u = 0; u < kStatsChunkVecs; ++u) {
+      const int vi = u * kConsumers + tid;
+      w[u] = vi < nv ? src[vi] : make_uint4(ni, ni, ni, ni);
+    }
+    __syncwarp();
+    if (lane == 0) ptx::mbar_arrive(&sm.empty[stg]);
+    ++c;
+    stats_add_chunk<LT, kStatsChunkVecs>(st, w);
   }
-  if (tid == 0) s_bad = 0;
-  __syncthreads();
-  // validate every draft token and gather the decision inputs of the first rows
-  for (int i = tid; i < k; i += NT) {
-    const int32_t y = __ldg(p.draft_tokens + D0 + i);
-    if (y < 0 || y >= V) {
-      atomicOr(&s_bad, 1);
-    } else if (i < kPreload) {
-      s_zy[i] = load_scalar(logits + (Q0 + i) * (int64_t)V, y);
-      s_qy[i] = __ldg(p.draft_probs + (D0 + i) * (int64_t)V + y);
-      s_u[i] = __ldg(p.accept_u + D0 + i);
-    }
-  }
-  __syncthreads();
-
-  // ---- reductions across the cluster -----------------------------------------------
-  // ff total over the CTA (per-thread values), every CTA's total gathered into s_tot,
-  // and their sum in rank order
-  auto cluster_total = [&](ff a) -> ff {
-    for (int o = 16; o > 0; o >>= 1) a = ff_add(a, ff_shfl_xor(a, o));
-    if (lane == 0) s_wst[warp].s = a;
-    __syncthreads();
-    if (tid == 0) {
-      ff t = {0.0f, 0.0f};
-      for (int w = 0; w < NW; ++w) t = ff_add(t, s_wst[w].s);
-      s_pub[xslot].s = t;
-    }
-    cluster.sync();
-    if (tid < C) s_tot[tid] = cluster.map_shared_rank(&s_pub[xslot], tid)->s;
-    __syncthreads();
-    ff t = {0.0f, 0.0f};
-    for (int q = 0; q < C; ++q) t = ff_add(t, s_tot[q]);
-    xslot ^= 1;
-    return t;
-  };
-  // double-float sum of f(element) over this thread's vectors of a row, in vector order; w[u] holds
-  // the vector u rounds ahead of the current one
-  auto thread_sum = [&](const LT *row, auto &&f) -> ff {
-    ff acc = {0.0f, 0.0f};
-    uint4 w[kZAhead];
-#pragma unroll
-    for (int u = 0; u < kZAhead; ++u) {
-      const int64_t vi = vlo + tid + (int64_t)u * NT;
-      if (vi < vhi) w[u] = load_vec<LT>(row, vi, V, vec_z);
-    }
-#pragma unroll 1
-    for (int64_t vi = vlo + tid; vi < vhi; vi += NT) {
-      const uint4 cur = w[0];
-#pragma unroll
-      for (int u = 0; u + 1 < kZAhead; ++u) w[u] = w[u + 1];
-      const int64_t vn = vi + (int64_t)kZAhead * NT;
-      if (vn < vhi) w[kZAhead - 1] = load_vec<LT>(row, vn, V, vec_z);
-      ff t[E];
-#pragma unroll
-      for (int i = 0; i < E; ++i) t[i] = f(cur, i);
-      acc = ff_add_pos(acc, ff_tree_pos<E>(t));
-    }
-    return acc;
-  };
-  // double-float normaliser of a row (re-streamed); m is the row's exact max
-  auto row_Zff = [&](const LT *row, float m) -> ff {
-    return cluster_total(thread_sum(row, [&](const uint4 &w, int i) {
-      const ff x = ff_two_sum(vec_elem<LT>(w, i), -m);
-      return ff_exp_nonpos(x.hi, x.lo, s_th, s_tl);
-    }));
-  };
-
-  // ---- the in-order walk (Eq. 1-2) -------------------------------------------
-  // The rows' statistics come from row_stats_kernel: warp w merges the slices of row i0 + w,
-  // then thread 0 takes the decisions of the batch in order; a decision inside the certified
-  // interval of the fp32 ratio stops it, the whole cluster recomputes that row's normaliser in
-  // double-float arithmetic, and the walk resumes after it.
-  int L = k;
-  int err = s_bad ? WISP_DEV_BAD_TOKEN : 0;
-  float m = 0.0f;
-  ff Zff = {0.0f, 0.0f};
-  bool have_Zff = false;
-  bool done = err != 0;
-  const int nsl = p.slices;
-  for (int i0 = 0; i0 <= k && !done; i0 += NW) {
-    if (i0 + warp <= k) {
-      const RowStats rs = merge_parts(p.parts + (Q0 + i0 + warp) * (int64_t)nsl, nsl);
-      if (lane == 0) s_rows[warp] = rs;
-    }
-    __syncthreads();
-    int j = 0;
-    while (!done) {
-      if (tid == 0) {
-        // state: 0 batch exhausted, 1 bonus row reached, 2 rejected, 3 bad row, 4 uncertain
-        int state = 0, jj = j;
-        Decide d;
-        d.flag = 0;
-        for (; jj < NW && i0 + jj <= k; ++jj) {
-          const int i = i0 + jj;
-          const RowStats rs = s_rows[jj];
-          const float mi = rs.m;
-          const ff Z = rs.s;
-          if (!(mi > -INFINITY) || !(mi < INFINITY) || !(Z.hi > 0.0f) || !(Z.hi < INFINITY) || !(rs.A >= 0.0f)) {
-            state = 3;
-            break;
-          }
-          if (i == k) {
-            state = 1;  // every draft token accepted
-            break;
-          }
-          if (i < kPreload) {
-            d.zy = s_zy[i];
-            d.qy = s_qy[i];
-            d.u = s_u[i];
-          } else {
-            const int32_t y = __ldg(p.draft_tokens + D0 + i);
-            d.zy = load_scalar(logits + (Q0 + i) * (int64_t)V, y);
-            d.qy = __ldg(p.draft_probs + (D0 + i) * (int64_t)V + y);
-            d.u = __ldg(p.accept_u + D0 + i);
-          }
-          if (!(d.qy >= 0.0f)) {
-            state = 3;
-            break;
-          }
-          if (d.qy == 0.0f) continue;  // a = 1: accepted
-          if (!(d.zy > -INFINITY)) {  // a masked token: p(y) = 0 exactly, accepted only if u = 0
-            if (d.u <= 0.0f) continue;
-            state = 2;
-            break;
-          }
-          // certified relative error of Z (see RowStats) and of the ratio p(y)/q(y)
-          // terms: one exp error per element and per rescale on its way (thread, CTA, row), three
-          // roundings in the argument (z - m, log2 e, the product) of every element and every
-          // rescale, the 32-term pairwise sums; the decision's own exp and ratio on top
-          const float x = d.zy - mi;
-          // outside the range of the fp32 ratio (2^x flushes to zero below 2^-126, a subnormal q(y)
-          // loses bits): decide in double precision
-          if (x * kLog2e < -126.0f || d.qy < FLT_MIN) {
-            state = 4;
-            break;
-          }
-          const float dz = 1.05f * ((float)(rs.nres + 2) * kEx2RelErr + 3.0f * 0x1p-24f * (mi - rs.mfirst) +
-                                    3.0f * 0x1p-24f * (rs.A / Z.hi) + 6.0f * 0x1p-24f) +
-                           1e-12f;
-          const float dr = dz + 1.05f * (kEx2RelErr + 3.0f * 0x1p-24f * fabsf(x) + 4.0f * 0x1p-24f);
-          const float ratio = ex2_approx(x * kLog2e) / (Z.hi * d.qy);
-          const float lo = fminf(1.0f, ratio * (1.0f - dr)), hi = fminf(1.0f, ratio * (1.0f + dr));
-          if (d.u <= lo) continue;
-          state = d.u > hi ? 2 : 4;
-          break;
-        }
-        s_walk[0] = state;
-        s_walk[1] = jj;
-        s_dec = d;
-      }
-      __syncthreads();
-      const int state = s_walk[0], jj = s_walk[1];
-      if (state == 0) break;  // next batch
-      if (state == 3) {
-        err = WISP_DEV_BAD_PROB;
-        done = true;
-      } else if (state == 1 || state == 2) {
-        L = i0 + jj;
-        m = s_rows[jj].m;
-        done = true;
-      } else {
-        // inside the certified interval: decide with the double-float normaliser
-        const int i = i0 + jj;
-        const float mi = s_rows[jj].m;
-        const ff zf = row_Zff(logits + (Q0 + i) * (int64_t)V, mi);
-        if (tid == 0) {
-          const Decide d = s_dec;
-          // p(y) / q(y) in double precision: z(y) - m is exact as a double, and neither p(y) nor a
-          // subnormal q(y) leaves the double range
-          const double ratio = exp((double)d.zy - (double)mi) / (ff_to_double(zf) * (double)d.qy);
-          s_walk[0] = (double)d.u <= fmin(1.0, ratio) ? 0 : 1;
-        }
-        __syncthreads();
-        if (s_walk[0] == 1) {
-          L = i;
-          m = mi;
-          Zff = zf;
-          have_Zff = true;
-          done = true;
-        } else {
-          j = jj + 1;  // accepted: resume the walk after this row
-        }
-      }
-      __syncthreads();  // s_walk / s_dec are rewritten by the next round
+  const RowStats ws = warp_merge(st);
+  if (lane == 0) sm.wst[warp] = ws;
+  cbar(sm, ph, p);
+  if (warp == 0) {
+    RowStats q;
+    stats_init(q);
+    if (lane < kCW) q = sm.wst[lane];
+    const RowStats cs = warp_merge(q);
+    if (lane == 0) {
+      it.sp.m = cs.m;
+      it.sp.s_hi = cs.s.hi;
+      it.sp.s_lo = cs.s.lo;
+      it.sp.A = cs.A;
+      it.sp.mfirst = cs.mfirst;
+      it.sp.nres = cs.nres;
+      it.sp.pad[0] = it.sp.pad[1] = 0;
     }
   }
+}
 
-  if (err) {
-    if (rank == 0 && tid == 0) {
-      report(p.status, err, p.request_ids, r);
-      p.accepted_len[r] = -1;
-      p.next_token[r] = -1;
-    }
-    cluster.sync();
-    return;
+// Warp sum of one 64-bit value per lane as a U96 (the 32-bit halves summed separately).
+__device__ __forceinline__ U96 warp_sum_u64(unsigned long long x) {
+  unsigned long long lo = x & 0xFFFFFFFFull, hi = x >> 32;
+  for (int o = 16; o > 0; o >>= 1) {
+    lo += __shfl_xor_sync(0xffffffffu, lo, o);
+    hi += __shfl_xor_sync(0xffffffffu, hi, o);
   }
+  U96 r = u96_zero();
+  r.lo = lo;
+  u96_add(r, hi << 32);
+  r.hi += (unsigned)(hi >> 32);
+  return r;
+}
+// Warp sum of non-negative double-float values (same-sign addition: no cancellation).
+__device__ __forceinline__ ff ff_add_pos(ff a, ff b) {
+  ff s = ff_two_sum(a.hi, b.hi);
+  s.lo = __fadd_rn(s.lo, __fadd_rn(a.lo, b.lo));
+  return ff_fast_two_sum(s.hi, s.lo);
+}
+__device__ __forceinline__ ff ff_warp_sum_pos(ff a) {
+  for (int o = 16; o > 0; o >>= 1) a = ff_add_pos(a, ff_shfl_xor(a, o));
+  return a;
+}
 
-  // ---- the extra token (Eq. 3) --------------------------------------------------
-  const LT *row = logits + (Q0 + L) * (int64_t)V;
-  const float *qrow = p.draft_probs + (D0 + L) * (int64_t)V;
-  bool residual = L < k;
-  // exp(u - m) of row L for the bf16 values u of the table's range
-  // (only for rows much longer than the table)
-  ff *s_etab = std::is_same<LT, uint16_t>::value && V >= kExpTabMinV ? s_tile + rounds * NW : nullptr;
-  if (s_etab) {
-#pragma unroll 2
-    for (int idx = tid; idx < kExpTabSize; idx += NT) {
-      const float u = bf16_bits_to_float(exp_tab_bits(idx));
-      s_etab[idx] = u > m ? ff{0.0f, 0.0f} : draw_weight(u, m, false, 0.0f, ff{}, s_th, s_tl);  // u > m never occurs
-    }
-    __syncthreads();
-  }
-  if (residual && !have_Zff)
-    Zff = cluster_total(thread_sum(row, [&](const uint4 &w, int i) { return elem_exp<LT>(w, i, m, s_etab, s_th, s_tl); }));
-  ff S = {0.0f, 0.0f};
-  for (;;) {
-    ff run = {0.0f, 0.0f};
-    // the row's and the draft's vectors of round rd + u in w[u], q[u]
-    uint4 w[kSweepAhead];
-    float q[kSweepAhead][E];
-    auto load_round = [&](int rd, uint4 &wv, float (&qv)[E]) {
-      const int64_t vi = vlo + (int64_t)rd * NT + tid;
-      if (rd < rounds && vi < vhi) {
-        wv = load_vec<LT>(row, vi, V, vec_z);
-        if (residual) {
-          load_q<E>(qrow, vi * E, V, vec_q, qv);
-        } else {
-#pragma unroll
-          for (int i = 0; i < E; ++i) qv[i] = 0.0f;
-        }
-      }
-    };
-#pragma unroll
-    for (int u = 0; u < kSweepAhead; ++u) load_round(u, w[u], q[u]);
-#pragma unroll 1
-    for (int rd = 0; rd < rounds; ++rd) {
-      const uint4 cw = w[0];
-      float cq[E];
-#pragma unroll
-      for (int i = 0; i < E; ++i) cq[i] = q[0][i];
-#pragma unroll
-      for (int u = 0; u + 1 < kSweepAhead; ++u) {
-        w[u] = w[u + 1];
-#pragma unroll
-        for (int i = 0; i < E; ++i) q[u][i] = q[u + 1][i];
-      }
-      load_round(rd + kSweepAhead, w[kSweepAhead - 1], q[kSweepAhead - 1]);
-      const int64_t vi = vlo + (int64_t)rd * NT + tid;
-      ff part = {0.0f, 0.0f};
-      if (vi < vhi) {
-        ff t[E];
-#pragma unroll
-        for (int i = 0; i < E; ++i) t[i] = weight_from(elem_exp<LT>(cw, i, m, s_etab, s_th, s_tl), residual, cq[i], Zff);
-        part = ff_tree_pos<E>(t);
-      }
-      for (int o = 16; o > 0; o >>= 1) part = ff_add_pos(part, ff_shfl_xor(part, o));
-      if (lane == 0) s_tile[rd * NW + warp] = part;
-      run = ff_add_pos(run, part);
-    }
-    // run is the warp's sum over all rounds (same value in every lane): count it once
-    if (lane != 0) run = {0.0f, 0.0f};
-    S = cluster_total(run);
-    if (residual && !(S.hi > 0.0f)) {
-      residual = false;  // the residual has no mass (only through rounding): draw from p_L instead
+// Draw item: slice of row L in chunks of 256 vectors.  The warps take chunks in two groups (warps
+// 0-3 the even chunks of the item, 4-7 the odd ones); in its chunk a warp owns 64 consecutive
+// vectors (a tile, two per lane), and the other group only waits for the chunk and releases it.
+// Per element the exact weight e = round(2^56 exp(z - m)); after a rejection also the sign of
+// p - q, settled with the fp32 normaliser and its certified bound where possible (p > q: e and q go
+// into E_P and Q_P; p <= q: no mass), else kept for the finisher.  Sums per tile (written to the
+// tile records) and per slice.
+template <typename LT>
+__device__ void c_draw(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint32_t &ph, const AcceptParams &p) {
+  constexpr int E = LTraits<LT>::E;
+  constexpr int TV = kDrawTile;  // vectors per tile
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int grp = warp / (kCW / 2), wi = warp % (kCW / 2);
+  const bool residual = it.resid != 0;
+  const RowRec rec = it.rec;
+  // Z lies in [z_hi (1 - dz), z_hi (1 + dz)]; margins of 2^-20 cover the fp32 roundings of the tests
+  const float zhi = rec.z_hi * (1.0f + rec.dz + 0x1p-20f);
+  const float zlo = rec.z_hi * (1.0f - rec.dz - 0x1p-20f);
+  TileRec *trec = p.tiles + (int64_t)it.r * p.ntiles;
+  U96 ea = u96_zero(), ep = u96_zero();
+  ff qp = {0.0f, 0.0f};
+  for (int j = 0; j < it.nchunks; ++j) {
+    const int stg = c % kStages;
+    if (!wait_bar(&sm.full[stg], (c / kStages) & 1, sm, p)) return;
+    const int64_t cv0 = it.v0 + (int64_t)j * kDrawChunk;
+    if ((j & 1) != grp) {  // the other group's chunk
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(&sm.empty[stg]);
+      ++c;
       continue;
     }
-    break;
-  }
-
-  // which CTA holds the crossing of u * S (every CTA computes the same answer)
-  if (tid == 0) {
-    const ff thr = ff_mul_f(S, __ldg(p.sample_u + r));
-    ff run = {0.0f, 0.0f};
-    int owner = -1, last_pos = -1;
-    ff local = thr;
-    for (int q = 0; q < C; ++q) {
-      const ff nxt = ff_add(run, s_tot[q]);
-      if (s_tot[q].hi > 0.0f) last_pos = q;
-      if (owner < 0 && ff_gt(nxt, thr)) {
-        owner = q;
-        local = ff_add(thr, ff_neg(run));
-      }
-      run = nxt;
-    }
-    s_owner = owner >= 0 ? owner : last_pos;
-    s_take_last = owner >= 0 ? 0 : 1;
-    s_thr = local;
-  }
-  __syncthreads();
-  const int owner = s_owner;
-  if (rank == owner && warp == 0) {
-    // tile entries (round, warp) are in token order: find the one holding the crossing
-    const int n_ent = rounds * NW;
-    bool take_last = s_take_last != 0;
-    const ff thr = s_thr;
-    int entry = -1;
-    ff before = {0.0f, 0.0f};
-    if (!take_last) {
-      ff base = {0.0f, 0.0f};
-      for (int e0 = 0; e0 < n_ent && entry < 0; e0 += 32) {
-        const ff v = e0 + lane < n_ent ? s_tile[e0 + lane] : ff{0.0f, 0.0f};
-        ff incl = v;
-        for (int d = 1; d < 32; d <<= 1) {
-          const ff o = ff_shfl_up(incl, d);
-          if (lane >= d) incl = ff_add(incl, o);
-        }
-        incl = ff_add(base, incl);
-        ff excl = ff_shfl_up(incl, 1);
-        if (lane == 0) excl = base;
-        const unsigned hit = __ballot_sync(0xffffffffu, e0 + lane < n_ent && ff_gt(incl, thr));
-        if (hit) {
-          const int l0 = __ffs(hit) - 1;
-          entry = e0 + l0;
-          before = {__shfl_sync(0xffffffffu, excl.hi, l0), __shfl_sync(0xffffffffu, excl.lo, l0)};
-        }
-        base = {__shfl_sync(0xffffffffu, incl.hi, 31), __shfl_sync(0xffffffffu, incl.lo, 31)};
-      }
-      if (entry < 0) take_last = true;  // rounding left no crossing inside this CTA
-    }
-    if (take_last) {
-      entry = -1;
-      for (int e0 = ((n_ent - 1) / 32) * 32; e0 >= 0 && entry < 0; e0 -= 32) {
-        const bool pos = e0 + lane < n_ent && s_tile[e0 + lane].hi > 0.0f;
-        const unsigned b = __ballot_sync(0xffffffffu, pos);
-        if (b) entry = e0 + 31 - __clz(b);
-      }
-    }
-    if (entry >= 0) {
-      // re-derive the tile's weights: lane sums, inclusive scan, then one lane's elements
-      const int rd = entry / NW, ww = entry % NW;
-      const int64_t vi = vlo + (int64_t)rd * NT + ww * 32 + lane;
-      float q[E];
-      ff wts[E];
-      ff lsum = {0.0f, 0.0f};
+    const char *sb = ring + (size_t)stg * kStageBytes;
+    uint4 w[2];
+    float q[2][E];
+    bool have[2];
 #pragma unroll
-      for (int i = 0; i < E; ++i) wts[i] = {0.0f, 0.0f};
-      if (vi < vhi) {
-        const uint4 w = load_vec<LT>(row, vi, V, vec_z);
+    for (int h = 0; h < 2; ++h) {
+      const int loc = wi * TV + h * 32 + lane;  // vector within the chunk
+      have[h] = cv0 + loc < it.v1;
+      w[h] = have[h] ? reinterpret_cast<const uint4 *>(sb)[loc] : make_uint4(0, 0, 0, 0);
+#pragma unroll
+      for (int i = 0; i < E; ++i) q[h][i] = 0.0f;
+      if (have[h] && residual) {
+        const float4 *qs = reinterpret_cast<const float4 *>(sb + kQOffset) + (size_t)loc * (E / 4);
+#pragma unroll
+        for (int x = 0; x < E / 4; ++x) {
+          const float4 t = qs[x];
+          q[h][4 * x] = t.x;
+          q[h][4 * x + 1] = t.y;
+          q[h][4 * x + 2] = t.z;
+          q[h][4 * x + 3] = t.w;
+        }
+      }
+    }
+    __syncwarp();
+    if (lane == 0) ptx::mbar_arrive(&sm.empty[stg]);
+    ++c;
+    unsigned long long sa = 0, sp = 0;
+    ff tq = {0.0f, 0.0f}, tq2 = {0.0f, 0.0f};
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      if (!have[h]) continue;
+      unsigned long long fx[E];
+      float fl[E];
+      weights<LT>(w[h], rec.m, sm, tab, fx, fl);
+      bool amb = false;
+#pragma unroll
+      for (int i = 0; i < E; ++i) {
+        sa += fx[i];
         if (residual) {
-          load_q<E>(qrow, vi * E, V, vec_q, q);
-        } else {
-#pragma unroll
-          for (int i = 0; i < E; ++i) q[i] = 0.0f;
+          const float qi = q[h][i];
+          const bool pos = qi >= 0.0f && fl[i] > qi * zhi;
+          if (pos) sp += fx[i];
+          if (i & 1)
+            ff_acc(tq2, pos ? qi : 0.0f);
+          else
+            ff_acc(tq, pos ? qi : 0.0f);
+          amb |= !pos && fl[i] > qi * zlo;  // neither certainly positive nor certainly without mass
         }
-#pragma unroll
+      }
+      if (amb) {
+        #pragma unroll
         for (int i = 0; i < E; ++i) {
-          wts[i] = weight_from(elem_exp<LT>(w, i, m, s_etab, s_th, s_tl), residual, q[i], Zff);
-          lsum = ff_add(lsum, wts[i]);
+          const float qi = q[h][i];
+          if (!(qi >= 0.0f && fl[i] > qi * zhi) && fl[i] > qi * zlo) {
+            const int a = atomicAdd(&sm.amb_n, 1);
+            if (a < kAmbPerSlice) {
+              sm.amb[a].e = fx[i];
+              sm.amb[a].q = qi;
+              sm.amb[a].v = (int)((cv0 + wi * TV + h * 32 + lane) * E + i);
+            }
+          }
         }
       }
-      const ff rem = ff_add(thr, ff_neg(before));
-      ff incl = lsum;
-      for (int d = 1; d < 32; d <<= 1) {
-        const ff o = ff_shfl_up(incl, d);
-        if (lane >= d) incl = ff_add(incl, o);
+    }
+    if (residual) tq = ff_add_pos(tq, tq2);
+    // the warp's tile: its sums, warp-wide, into the tile records
+    const U96 A_ = warp_sum_u64(sa), P_ = residual ? warp_sum_u64(sp) : u96_zero();
+    const ff Q_ = residual ? ff_warp_sum_pos(tq) : ff{0.0f, 0.0f};
+    if (p.tile_vecs && lane == 0 && cv0 + wi * TV < it.v1) {
+      TileRec r;
+      r.e_all = u96_to_double(A_);
+      r.e_p = u96_to_double(P_);
+      r.q_hi = Q_.hi;
+      r.q_lo = Q_.lo;
+      trec[(cv0 + wi * TV) / TV] = r;
+    }
+    u96_add(ea, A_);
+    u96_add(ep, P_);
+    qp = ff_add_pos(qp, Q_);
+  }
+  // slice totals (each warp holds its own, identical in its lanes)
+  if (lane == 0) {
+    sm.red[0][0][warp] = ea;
+    sm.red[0][1][warp] = ep;
+    sm.qred[0][warp] = qp;
+  }
+  cbar(sm, ph, p);
+  if (tid == 0) {
+    U96 a = u96_zero(), b = u96_zero();
+    ff t = {0.0f, 0.0f};
+    for (int x = 0; x < kCW; ++x) {
+      u96_add(a, sm.red[0][0][x]);
+      u96_add(b, sm.red[0][1][x]);
+      t = ff_add_pos(t, sm.qred[0][x]);
+    }
+    it.ea = a;
+    it.ep = b;
+    it.qp = t;
+    const int na = sm.amb_n;
+    it.n_amb = na;
+    for (int x = 0; x < na && x < kAmbPerSlice; ++x) it.amb[x] = sm.amb[x];
+    __threadfence();  // the tile records before the keeper's completion count
+  }
+}
+
+// Finish item: the tile holding the crossing of u * total (Eq. 3), chunk by chunk; per thread the
+// exact weight of its vector, a consumer-wide scan in token order, and the element within the
+// thread holding the crossing; or, with take_last, the last element with weight.  Writes the outputs.
+template <typename LT>
+__device__ void c_finish(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint32_t &ph, const AcceptParams &p) {
+  constexpr int E = LTraits<LT>::E;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool residual = it.resid != 0;
+  double carry = 0.0;
+  const double thr = it.thr;
+  const bool tl = it.take_last != 0;  // no crossing to look for: the last element with weight
+  bool found = false;
+  int64_t last_vec = -1;              // (thread 0) the last vector with weight
+  for (int j = 0; j < it.nchunks; ++j) {
+    const int stg = c % kStages;
+    if (!wait_bar(&sm.full[stg], (c / kStages) & 1, sm, p)) return;
+    const char *sb = ring + (size_t)stg * kStageBytes;
+    const int64_t cv0 = it.v0 + (int64_t)j * kDrawChunk;
+    const bool have = cv0 + tid < it.v1;
+    uint4 w = make_uint4(0, 0, 0, 0);
+    float q[E];
+#pragma unroll
+    for (int i = 0; i < E; ++i) q[i] = 0.0f;
+    if (have) {
+      w = reinterpret_cast<const uint4 *>(sb)[tid];
+      if (residual) {
+        const float4 *qs = reinterpret_cast<const float4 *>(sb + kQOffset) + (size_t)tid * (E / 4);
+#pragma unroll
+        for (int h = 0; h < E / 4; ++h) {
+          const float4 t = qs[h];
+          q[4 * h] = t.x;
+          q[4 * h + 1] = t.y;
+          q[4 * h + 2] = t.z;
+          q[4 * h + 3] = t.w;
+        }
       }
-      ff excl = ff_shfl_up(incl, 1);
-      if (lane == 0) excl = {0.0f, 0.0f};
-      int l0 = -1;
-      if (!take_last) {
-        const unsigned hit = __ballot_sync(0xffffffffu, ff_gt(incl, rem));
-        if (hit) l0 = __ffs(hit) - 1;
-      }
-      const bool last_mode = take_last || l0 < 0;
-      if (last_mode) {
-        const unsigned b = __ballot_sync(0xffffffffu, lsum.hi > 0.0f);
-        l0 = b ? 31 - __clz(b) : -1;
-      }
-      if (l0 >= 0 && lane == l0) {
-        const ff r2 = ff_add(rem, ff_neg(excl));
-        ff acc = {0.0f, 0.0f};
-        int tok = -1, last = -1;
+    }
+    __syncwarp();
+    if (lane == 0) ptx::mbar_arrive(&sm.empty[stg]);
+    ++c;
+    const double wv = have ? vec_weight<LT>(w, q, residual, it.rec.m, it.Zu, sm, tab) : 0.0;
+    double incl = wv;
+    for (int o = 1; o < 32; o <<= 1) {
+      const double t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (lane == 31) sm.dred[warp] = incl;
+    if (tid == 0) {
+      sm.first = INT32_MAX;
+      sm.lastpos = -1;
+    }
+    cbar(sm, ph, p);
+    double off = carry;
+    for (int x = 0; x < warp; ++x) off += sm.dred[x];
+    double total = carry;
+    for (int x = 0; x < kCW; ++x) total += sm.dred[x];
+    incl += off;
+    if (!tl && !found && incl > thr) atomicMin(&sm.first, tid);
+    if (wv > 0.0) atomicMax(&sm.lastpos, tid);
+    cbar(sm, ph, p);
+    if (!tl && !found && sm.first != INT32_MAX) {
+      if (tid == sm.first) {
+        // this thread's elements in order, with exact weights
+        unsigned long long fx[E];
+        float fl[E];
+        weights<LT>(w, it.rec.m, sm, tab, fx, fl);
+        const double r2 = thr - (incl - wv);
+        double acc = 0.0;
+        int tok = -1, lastv = -1;
+        #pragma unroll
         for (int i = 0; i < E; ++i) {
-          const int64_t v = vi * E + i;
-          if (v >= V) break;
-          if (wts[i].hi > 0.0f) last = (int)v;
-          acc = ff_add(acc, wts[i]);
-          if (!last_mode && ff_gt(acc, r2)) {
+          const int64_t v = (cv0 + tid) * E + i;
+          if (v >= p.V) break;
+          const double wt = weight_d(fx[i], q[i], residual, it.Zu);
+          if (wt > 0.0) lastv = (int)v;
+          acc += wt;
+          if (acc > r2) {
             tok = (int)v;
             break;
           }
         }
-        p.next_token[r] = tok >= 0 ? tok : last;
+        p.accepted_len[it.r] = it.i;
+        p.next_token[it.r] = tok >= 0 ? tok : lastv;
       }
-    } else if (lane == 0) {
-      p.next_token[r] = -1;  // no element with mass: cannot happen for a finite row
+      found = true;
+    }
+    if (tid == 0 && sm.lastpos >= 0) last_vec = cv0 + sm.lastpos;
+    carry = total;
+    cbar(sm, ph, p);  // sm.first / sm.lastpos / sm.dred are rewritten by the next chunk
+  }
+  if (!found && tid == 0) {
+    // rounding left no crossing in the tile (or take_last): the last element with weight
+    int tok = -1;
+    if (last_vec >= 0) {
+      const LT *row = static_cast<const LT *>(p.logits) + (it.Q0 + it.i) * (int64_t)p.V;
+      const float *qrow = p.draft_probs + (it.D0 + it.i) * (int64_t)p.V;
+      const uint4 w = load_vec<LT>(row, last_vec, p.V, p.vec_z != 0);
+      float q[E];
+      #pragma unroll
+      for (int i = 0; i < E; ++i) q[i] = 0.0f;
+      if (residual) load_q<E>(qrow, last_vec * E, p.V, p.vec_q != 0, q);
+      unsigned long long fx[E];
+      float fl[E];
+      weights<LT>(w, it.rec.m, sm, tab, fx, fl);
+      #pragma unroll
+      for (int i = 0; i < E; ++i) {
+        const int64_t v = last_vec * E + i;
+        if (v < p.V && weight_d(fx[i], q[i], residual, it.Zu) > 0.0) tok = (int)v;
+      }
+    }
+    p.accepted_len[it.r] = it.i;
+    p.next_token[it.r] = tok;
+  }
+}
+
+}  // namespace
+
+namespace {
+
+// ---- the keeper (warp 9): completions, row decisions, L, the draw's crossing search ------------
+struct DecIn {
+  float zy, qy, u;
+};
+
+// The decision row i scores (Eq. 1 for draft token i + 1), taken by one thread from the row's
+// merged statistics: ROW_ACCEPT / ROW_REJECT when u lies outside the certified interval of the
+// fp32 ratio p(y) / q(y), ROW_UNCERTAIN otherwise (decided with the exact normaliser).
+template <typename LT>
+__device__ int decide(const AcceptParams &p, const RowRec &rec, int64_t R, int64_t D0, int i, DecIn &d) {
+  const int32_t y = __ldg(p.draft_tokens + D0 + i);
+  if (y < 0 || y >= p.V) return ROW_BAD_TOKEN;
+  const LT *row = static_cast<const LT *>(p.logits) + R * (int64_t)p.V;
+  d.zy = load_scalar(row, y);
+  d.qy = __ldg(p.draft_probs + (D0 + i) * (int64_t)p.V + y);
+  d.u = __ldg(p.accept_u + D0 + i);
+  const float zy = d.zy, qy = d.qy, u = d.u;
+  if (!(qy >= 0.0f)) return ROW_BAD_PROB;
+  if (qy == 0.0f) return ROW_ACCEPT;                                   // a = 1
+  if (!(zy > -INFINITY)) return u <= 0.0f ? ROW_ACCEPT : ROW_REJECT;  // p(y) = 0 exactly
+  const float x = zy - rec.m;
+  // outside the range of the fp32 ratio (2^x flushes to zero below 2^-126, a subnormal q(y) loses
+  // bits): the exact path, in double precision
+  if (x * kLog2e < -126.0f || qy < FLT_MIN) return ROW_UNCERTAIN;
+  // the decision's own exp (error and argument roundings) and ratio roundings on top of Z's bound
+  const float dr = rec.dz + 1.05f * (kEx2RelErr + 3.0f * 0x1p-24f * fabsf(x) + 4.0f * 0x1p-24f);
+  const float ratio = ex2_approx(x * kLog2e) / (rec.z_hi * qy);
+  const float lo = fminf(1.0f, ratio * (1.0f - dr)), hi = fminf(1.0f, ratio * (1.0f + dr));
+  if (u <= lo) return ROW_ACCEPT;
+  if (u > hi) return ROW_REJECT;
+  return ROW_UNCERTAIN;
+}
+
+// Is request r's accepted length now known?  The codes of rows 0..k are read in order (one lane
+// each): the first rejection gives L, a valid bonus row L = k, a bad row an error, an unknown row
+// means not yet.  The first warp to see the answer claims the request and queues it for its draw
+// (or records its error).
+__device__ void try_determine(const AcceptParams &p, int r, int k, int64_t Q0) {
+  const int lane = threadIdx.x & 31;
+  int L = -1, err = 0;
+  for (int j0 = 0; j0 <= k; j0 += 32) {
+    const int j = j0 + lane;
+    const int c = j <= k ? ld_vol(p.row_code + Q0 + j) : ROW_ACCEPT;
+    const unsigned nonacc = __ballot_sync(0xffffffffu, c != ROW_ACCEPT);
+    if (nonacc == 0) continue;
+    const int l0 = __ffs(nonacc) - 1;
+    const int c0 = __shfl_sync(0xffffffffu, c, l0);
+    if (c0 == ROW_UNKNOWN) return;
+    if (c0 == ROW_REJECT)
+      L = j0 + l0;
+    else if (c0 == ROW_BONUS)
+      L = k;
+    else
+      err = c0 == ROW_BAD_TOKEN ? WISP_DEV_BAD_TOKEN : WISP_DEV_BAD_PROB;
+    break;
+  }
+  if (L < 0 && !err) return;
+  if (lane != 0) return;
+  if (atomicCAS(p.req_claim + r, 0, 1) != 0) return;
+  atomicMin(p.req_rej + r, -1);  // every remaining statistics item of the request is skipped
+  if (err) {
+    report(p.status, err, p.request_ids, r);
+    p.accepted_len[r] = -1;
+    p.next_token[r] = -1;
+    __threadfence();
+    atomicAdd(&p.ctr->n_claimed, 1);
+    return;
+  }
+  st_vol(p.req_L + r, L);
+  __threadfence();
+  const int pos = atomicAdd(&p.ctr->q_reserve, 1);  // reserve a queue entry
+  st_vol(p.queue + pos, r);
+  __threadfence();
+  atomicAdd(&p.ctr->n_claimed, 1);  // after the queue entry: a CTA that sees every request claimed sees it
+}
+
+// Exact draw weight (units 2^-56) of vectors [a, b) of a row, by one warp alone (lanes stride), each
+// element's exp computed directly: the rare paths (an uncertain decision's normaliser, a slice
+// whose undecided elements overflowed its record).  q = nullptr: the weights exp(z - m) themselves.
+template <typename LT>
+__device__ double warp_range_weight(const AcceptParams &p, const Sm &sm, const LT *row, const float *qrow, float m,
+                                    double Zu, int64_t a, int64_t b) {
+  constexpr int E = LTraits<LT>::E;
+  const int lane = threadIdx.x & 31;
+  double acc = 0.0;
+  for (int64_t vi = a + lane; vi < b; vi += 32) {
+    const uint4 w = load_vec<LT>(row, vi, p.V, p.vec_z != 0);
+    float q[E];
+    #pragma unroll
+    for (int i = 0; i < E; ++i) q[i] = 0.0f;
+    if (qrow) load_q<E>(qrow, vi * E, p.V, p.vec_q != 0, q);
+    acc += vec_weight<LT>(w, q, qrow != nullptr, m, Zu, sm, Tab{nullptr, nullptr, nullptr});
+  }
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  return acc;
+}
+
+// A statistics item is complete: its slice record, the row's count; the warp that completes the
+// row merges its slices, takes the decision, checks the draft (at row 0), publishes the row's code
+// and tries to determine L.
+template <typename LT>
+__device__ void k_stats(const AcceptParams &p, Sm &sm, const Item &it) {
+  const int lane = threadIdx.x & 31;
+  int last = 0;
+  if (lane == 0) {
+    p.sparts[it.R * p.sslices + it.s] = it.sp;
+    __threadfence();
+    last = atomicAdd(&p.row_cnt[it.R], 1) == p.sslices - 1;
+  }
+  if (!__shfl_sync(0xffffffffu, last, 0)) return;
+  __threadfence();
+  const int r = it.r, i = it.i, k = it.k;
+  RowStats q;
+  stats_init(q);
+  if (lane < p.sslices) {
+    const SlicePart *sp = p.sparts + it.R * p.sslices + lane;
+    q.m = __ldcg(&sp->m);
+    q.s.hi = __ldcg(&sp->s_hi);
+    q.s.lo = __ldcg(&sp->s_lo);
+    q.A = __ldcg(&sp->A);
+    q.mfirst = __ldcg(&sp->mfirst);
+    q.nres = __ldcg(&sp->nres);
+  }
+  const RowStats rs = warp_merge(q);
+  RowRec rec;
+  rec.m = rs.m;
+  rec.z_hi = rs.s.hi;
+  rec.z_lo = rs.s.lo;
+  const bool ok = rs.m > -INFINITY && rs.m < INFINITY && rs.s.hi > 0.0f && rs.s.hi < INFINITY && rs.A >= 0.0f;
+  rec.dz = ok ? z_bound(rs) : 0.0f;
+  DecIn d{0.0f, 0.0f, 0.0f};
+  int code = 0;
+  if (lane == 0) code = !ok ? ROW_BAD_PROB : i == k ? ROW_BONUS : decide<LT>(p, rec, it.R, it.D0, i, d);
+  code = __shfl_sync(0xffffffffu, code, 0);
+  // the whole draft is validated when row 0 (which the rule always reads) is finished
+  if (i == 0 && k > 0) {
+    bool bad = false;
+    for (int j = lane; j < k; j += 32) {
+      const int32_t y = __ldg(p.draft_tokens + it.D0 + j);
+      bad |= y < 0 || y >= p.V;
+    }
+    if (__any_sync(0xffffffffu, bad)) code = ROW_BAD_TOKEN;
+  }
+  if (code == ROW_UNCERTAIN) {
+    const LT *row = static_cast<const LT *>(p.logits) + it.R * (int64_t)p.V;
+    const int64_t nvec = (p.V + LTraits<LT>::E - 1) / LTraits<LT>::E;
+    const double Zu = warp_range_weight<LT>(p, sm, row, nullptr, rec.m, 0.0, 0, nvec);
+    d.zy = __shfl_sync(0xffffffffu, d.zy, 0);
+    d.qy = __shfl_sync(0xffffffffu, d.qy, 0);
+    d.u = __shfl_sync(0xffffffffu, d.u, 0);
+    // p(y) / q(y) in double precision: z(y) - m is exact, and neither p(y) nor a subnormal q(y)
+    // leaves the double range
+    const double ratio = exp((double)d.zy - (double)rec.m) * 0x1p56 / (Zu * (double)d.qy);
+    code = (double)d.u <= fmin(1.0, ratio) ? ROW_ACCEPT : ROW_REJECT;
+  }
+  if (lane == 0) {
+    p.row_rec[it.R] = rec;
+    __threadfence();
+    st_vol(p.row_code + it.R, code);
+    if (code == ROW_REJECT) atomicMin(p.req_rej + r, i);
+  }
+  __syncwarp();
+  fence_sc();  // this code before the codes read next (against the keeper of another row)
+  try_determine(p, r, k, it.Q0);
+}
+
+// Post a finish task to this CTA's producer (bounded wait for room).
+__device__ bool post_finish(Sm &sm, const FinTask &f, const AcceptParams &p) {
+  const long long t0 = clock64();
+  while (vload(sm.fq_tail) - vload(sm.fq_head) >= kFinQ) {
+    if (vload(sm.abort_) || clock64() - t0 > kWaitCycles) {
+      if (atomicExch(&sm.abort_, 1) == 0) report(p.status, WISP_DEV_TIMEOUT, nullptr, -1);
+      return false;
     }
   }
-  if (rank == 0 && tid == 0) {
-    p.accepted_len[r] = L;
-    if (owner < 0) p.next_token[r] = -1;
+  const int t = sm.fq_tail;
+  sm.fq[t % kFinQ] = f;
+  __threadfence_block();
+  vstore(sm.fq_tail, t + 1);
+  return true;
+}
+
+// A draw item is complete: its slice record and the request's count.  The warp that completes the
+// request: exact normaliser (the slices' sums of exp(z - m)), residual mass per slice, the slice
+// holding the crossing of u * total (Eq. 3), the tile within it (from the tile records); the token
+// within the tile is found by a finish item on this CTA's consumers.
+template <typename LT>
+__device__ void k_draw(const AcceptParams &p, Sm &sm, const Item &it) {
+  constexpr int E = LTraits<LT>::E;
+  const int lane = threadIdx.x & 31;
+  const int Sd = p.dslices, r = it.r;
+  int last = 0;
+  if (lane == 0) {
+    DrawPart *out = p.dparts + (int64_t)r * Sd + it.s;
+    out->e_all = it.ea;
+    out->e_p = it.ep;
+    out->q_hi = it.qp.hi;
+    out->q_lo = it.qp.lo;
+    out->n_amb = it.n_amb;
+    for (int x = 0; x < it.n_amb && x < kAmbPerSlice; ++x) out->amb[x] = it.amb[x];
+    __threadfence();
+    last = atomicAdd(p.req_dcnt + r, 1) == Sd - 1;
   }
-  cluster.sync();  // no CTA leaves while another may still read its shared memory
+  if (!__shfl_sync(0xffffffffu, last, 0)) return;
+  __threadfence();
+  const int64_t nvec = (p.V + E - 1) / E;
+  const LT *row = static_cast<const LT *>(p.logits) + (it.Q0 + it.i) * (int64_t)p.V;
+  const float *qrow = p.draft_probs + (it.D0 + it.i) * (int64_t)p.V;
+  U96 ea = u96_zero(), ep = u96_zero();
+  double qp = 0.0;
+  int na = 0;
+  const DrawPart *dp = p.dparts + (int64_t)r * Sd + lane;
+  if (lane < Sd) {
+    ea.lo = __ldcg(&dp->e_all.lo);
+    ea.hi = __ldcg(&dp->e_all.hi);
+    ep.lo = __ldcg(&dp->e_p.lo);
+    ep.hi = __ldcg(&dp->e_p.hi);
+    qp = (double)__ldcg(&dp->q_hi) + (double)__ldcg(&dp->q_lo);
+    na = __ldcg(&dp->n_amb);
+  }
+  const double Zu = u96_to_double(u96_warp_sum(ea));
+  bool resid = it.resid != 0;
+  const double se = u96_to_double(ea);
+  double sd = se;
+  bool over = false;
+  if (resid) {
+    sd = u96_to_double(ep) - Zu * qp;
+    if (na > kAmbPerSlice) {
+      over = true;
+    } else {
+      for (int j = 0; j < na; ++j) sd += weight_d(__ldcg(&dp->amb[j].e), __ldcg(&dp->amb[j].q), true, Zu);
+    }
+  }
+  // slices with more undecided elements than their record holds: their mass by an exact pass
+  const unsigned ov = __ballot_sync(0xffffffffu, lane < Sd && over);
+  for (unsigned o = ov; o; o &= o - 1) {
+    const int d = __ffs(o) - 1;
+    const int64_t a = min(nvec, (int64_t)d * p.vpd), b = min(nvec, a + p.vpd);
+    const double t = warp_range_weight<LT>(p, sm, row, qrow, it.rec.m, Zu, a, b);
+    if (lane == d) sd = t;
+  }
+  // total in slice order (lane 0)
+  double S = 0.0;
+  for (int d = 0; d < Sd; ++d) S += __shfl_sync(0xffffffffu, sd, d);
+  if (resid && !(S > 0.0)) {
+    // the residual has no mass (only through rounding): draw from p_L instead
+    resid = false;
+    sd = se;
+    S = 0.0;
+    for (int d = 0; d < Sd; ++d) S += __shfl_sync(0xffffffffu, sd, d);
+  }
+  const double thr = (double)__ldg(p.sample_u + r) * S;
+  double run = 0.0, thr_d = 0.0;
+  int owner = -1, lastd = -1;
+  for (int d = 0; d < Sd; ++d) {
+    const double t = __shfl_sync(0xffffffffu, sd, d);
+    if (owner < 0 && run + t > thr) {
+      owner = d;
+      thr_d = thr - run;
+    }
+    run += t;
+    if (t > 0.0) lastd = d;
+  }
+  int take_last = owner < 0 ? 1 : 0;  // rounding left no crossing: the last token with mass
+  const int d = owner >= 0 ? owner : lastd;
+  if (d < 0) {  // no token has mass (cannot happen for a valid row)
+    if (lane == 0) {
+      p.accepted_len[r] = it.i;
+      p.next_token[r] = -1;
+    }
+    return;
+  }
+  const int64_t s0 = (int64_t)d * p.vpd, s1 = min(nvec, s0 + p.vpd);
+  FinTask f;
+  f.r = r;
+  f.i = it.i;
+  f.k = it.k;
+  f.resid = resid ? 1 : 0;
+  f.Q0 = it.Q0;
+  f.D0 = it.D0;
+  f.rec = it.rec;
+  f.Zu = Zu;
+  if (p.tile_vecs == 0) {
+    // no tile records (they would not fit): the finish item searches the whole slice
+    if (lane == 0) {
+      f.take_last = take_last;
+      f.v0 = s0;
+      f.v1 = s1;
+      f.thr = thr_d;
+      post_finish(sm, f, p);
+    }
+    return;
+  }
+  // the tile within slice d
+  const int64_t tlo = (int64_t)d * p.vpd / p.tile_vecs;
+  const int64_t thi = min((int64_t)p.ntiles, (min(nvec, (int64_t)(d + 1) * p.vpd) + p.tile_vecs - 1) / p.tile_vecs);
+  int64_t tile = -1;
+  double thr_t = thr_d;
+  const bool d_over = (ov >> d) & 1u;
+  const int nad = resid && !d_over ? __shfl_sync(0xffffffffu, na, d) : 0;
+  const DrawPart *dd = p.dparts + (int64_t)r * Sd + d;
+  const TileRec *tr = p.tiles + (int64_t)r * p.ntiles;
+  run = 0.0;
+  int64_t lastpos = -1;
+  for (int64_t t0 = tlo; t0 < thi && tile < 0; t0 += 32) {
+    const int64_t t = t0 + lane;
+    double w = 0.0;
+    if (t < thi) {
+      if (d_over) {
+        w = 0.0;  // filled below, one tile at a time, by the whole warp
+      } else if (resid) {
+        w = __ldcg(&tr[t].e_p) - Zu * ((double)__ldcg(&tr[t].q_hi) + (double)__ldcg(&tr[t].q_lo));
+        for (int j = 0; j < nad; ++j) {
+          const int64_t vt = (int64_t)(__ldcg(&dd->amb[j].v) / E) / p.tile_vecs;
+          if (vt == t) w += weight_d(__ldcg(&dd->amb[j].e), __ldcg(&dd->amb[j].q), true, Zu);
+        }
+      } else {
+        w = __ldcg(&tr[t].e_all);
+      }
+    }
+    if (d_over) {
+      // the slice's tile sums miss undecided elements: exact tile masses
+      for (int x = 0; x < 32 && t0 + x < thi; ++x) {
+        const int64_t tt = t0 + x;
+        const double m_ = warp_range_weight<LT>(p, sm, row, resid ? qrow : nullptr, it.rec.m, Zu,
+                                                tt * p.tile_vecs, min(nvec, (tt + 1) * p.tile_vecs));
+        if (lane == x) w = m_;
+      }
+    }
+    double incl = w;
+    for (int o = 1; o < 32; o <<= 1) {
+      const double u = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += u;
+    }
+    incl += run;
+    const unsigned pos = __ballot_sync(0xffffffffu, t < thi && w > 0.0);
+    if (pos) lastpos = t0 + 31 - __clz(pos);
+    if (!take_last) {
+      const unsigned hit = __ballot_sync(0xffffffffu, t < thi && incl > thr_d);
+      if (hit) {
+        const int l0 = __ffs(hit) - 1;
+        tile = t0 + l0;
+        thr_t = thr_d - __shfl_sync(0xffffffffu, incl - w, l0);
+      }
+    }
+    run = __shfl_sync(0xffffffffu, incl, 31);
+  }
+  if (tile < 0) {
+    tile = lastpos;
+    take_last = 1;
+  }
+  if (lane == 0) {
+    if (tile < 0) {
+      p.accepted_len[r] = it.i;
+      p.next_token[r] = -1;
+      return;
+    }
+    f.take_last = take_last;
+    f.v0 = tile * p.tile_vecs;
+    f.v1 = min(nvec, f.v0 + p.tile_vecs);
+    f.thr = thr_t;
+    post_finish(sm, f, p);
+  }
+}
+
+template <typename LT>
+__device__ void keeper(const AcceptParams &p, Sm &sm) {
+  const int lane = threadIdx.x & 31;
+  for (int n = 0;; ++n) {
+    const int slot = n % kItemSlots;
+    if (!wait_bar(&sm.res_ready[slot], (n / kItemSlots) & 1, sm, p)) return;
+    const Item &it = sm.item[slot];
+    const int kind = it.kind;
+    if (kind == WORK_EXIT) return;
+    if (kind == WORK_STATS) k_stats<LT>(p, sm, it);
+    if (kind == WORK_DRAW) k_draw<LT>(p, sm, it);
+    __syncwarp();
+    if (lane == 0) {
+      __threadfence_block();
+      vstore(sm.keeper_done, n + 1);  // after any finish task this item posted
+      ptx::mbar_arrive(&sm.iq_empty[slot]);
+    }
+    __syncwarp();
+  }
+}
+
+}  // namespace
+
+namespace {
+
+
+// ---- the producer (warp 8): next item, bulk copies into the ring ---------------------------------
+// Lane 0: the next work item of this CTA.  A finish task of this CTA first (it ends a request),
+// then draw tickets (their rows are still in L2), then the next statistics item in the level-major
+// order (skipping rows past a known rejection and rows of decided requests).  WORK_EXIT once every valid request is decided, every draw ticket taken and
+// this CTA has nothing pending; WORK_WAIT otherwise.
+template <typename LT>
+__device__ int pick(const AcceptParams &p, Sm &sm, Item &d, long long &idle_since, int issued, int &pend) {
+  constexpr int E = LTraits<LT>::E;
+  const int64_t nvec = (p.V + E - 1) / E;
+  AccCounters *c = p.ctr;
+  const int Sd = p.dslices;
+  if (vload(sm.abort_)) return WORK_EXIT;
+  const int fh = vload(sm.fq_head);
+  if (fh != vload(sm.fq_tail)) {
+    __threadfence_block();
+    const FinTask f = sm.fq[fh % kFinQ];
+    vstore(sm.fq_head, fh + 1);
+    d.kind = WORK_FINISH;
+    d.r = f.r;
+    d.i = f.i;
+    d.k = f.k;
+    d.s = 0;
+    d.resid = f.resid;
+    d.Q0 = f.Q0;
+    d.D0 = f.D0;
+    d.R = f.Q0 + f.i;
+    d.rec = f.rec;
+    d.thr = f.thr;
+    d.Zu = f.Zu;
+    d.take_last = f.take_last;
+    d.v0 = f.v0;
+    d.v1 = f.v1;
+    d.nchunks = (int)((d.v1 - d.v0 + kDrawChunk - 1) / kDrawChunk);
+    idle_since = -1;
+    return WORK_FINISH;
+  }
+  // draw tickets: one atomic increment of the head takes the next ticket.  A ticket taken past the
+  // entries reserved so far (a race with other producers) stays pending while this CTA goes on with
+  // statistics items; it is used once its entry exists, or lapses once every request is decided.
+  if (pend < 0 && ld_vol(&c->q_head) < ld_vol(&c->q_reserve) * Sd) pend = atomicAdd(&c->q_head, 1);
+  int r = -1;
+  if (pend >= 0 && pend < ld_vol(&c->q_reserve) * Sd) {
+    const long long t0 = clock64();
+    r = ld_vol(p.queue + pend / Sd);
+    while (r < 0) {  // the entry's keeper writes it right after reserving it
+      if (clock64() - t0 > kWaitCycles) {
+        if (atomicExch(&sm.abort_, 1) == 0) report(p.status, WISP_DEV_TIMEOUT, nullptr, -1);
+        return WORK_EXIT;
+      }
+      __nanosleep(64);
+      r = ld_vol(p.queue + pend / Sd);
+    }
+  }
+  if (r >= 0) {
+    const unsigned head = (unsigned)pend;
+    pend = -1;
+    __threadfence();
+    d.kind = WORK_DRAW;
+    d.r = r;
+    d.s = (int)(head % Sd);
+    d.i = ld_vol(p.req_L + r);
+    d.k = __ldg(p.draft_lens + r);
+    d.Q0 = __ldg(p.q_row_start + r);
+    d.D0 = __ldg(p.draft_start + r);
+    d.R = d.Q0 + d.i;
+    d.resid = d.i < d.k;
+    const RowRec *rr = p.row_rec + d.R;
+    d.rec.m = __ldcg(&rr->m);
+    d.rec.z_hi = __ldcg(&rr->z_hi);
+    d.rec.z_lo = __ldcg(&rr->z_lo);
+    d.rec.dz = __ldcg(&rr->dz);
+    d.v0 = min(nvec, (int64_t)d.s * p.vpd);
+    d.v1 = min(nvec, d.v0 + p.vpd);
+    d.nchunks = (int)((d.v1 - d.v0 + kDrawChunk - 1) / kDrawChunk);
+    idle_since = -1;
+    return WORK_DRAW;
+  }
+  const int n_items = __ldcg(&c->n_items);
+  while (ld_vol(&c->stats_next) < n_items) {
+    const int t = atomicAdd(&c->stats_next, 1);
+    if (t >= n_items) break;
+    const int2 ent = __ldcg(p.row_order + t / p.sslices);
+    const int r = ent.x, i = ent.y;
+    if (i > ld_vol(p.req_rej + r)) continue;  // past a rejection, or the request is decided
+    d.kind = WORK_STATS;
+    d.r = r;
+    d.i = i;
+    d.s = t % p.sslices;
+    d.k = __ldg(p.draft_lens + r);
+    d.Q0 = __ldg(p.q_row_start + r);
+    d.D0 = __ldg(p.draft_start + r);
+    d.R = d.Q0 + i;
+    d.resid = 0;
+    d.v0 = min(nvec, (int64_t)d.s * p.svps);
+    d.v1 = min(nvec, d.v0 + p.svps);
+    d.nchunks = (int)((d.v1 - d.v0 + kStatsChunk - 1) / kStatsChunk);
+    idle_since = -1;
+    return WORK_STATS;
+  }
+  if (ld_vol(&c->n_claimed) >= __ldcg(&c->n_valid)) {
+    fence_sc();
+    const int res = ld_vol(&c->q_reserve) * Sd;
+    if (pend >= res) pend = -1;  // no entry will ever hold this ticket
+    if (pend < 0 && vload(sm.keeper_done) == issued && ld_vol(&c->q_head) >= res &&
+        vload(sm.fq_head) == vload(sm.fq_tail))
+      return WORK_EXIT;
+  }
+  const long long now = clock64();
+  if (idle_since < 0) idle_since = now;
+  if (now - idle_since > kWaitCycles) {
+    if (atomicExch(&sm.abort_, 1) == 0) report(p.status, WISP_DEV_TIMEOUT, nullptr, -1);
+    return WORK_EXIT;
+  }
+  return WORK_WAIT;
+}
+
+// Copy chunk j of item `it` into a stage: bulk copies when the rows are 16-byte aligned (z at the
+// stage start, q at kQOffset), else the warp's own loads (padding with -inf / 0 past V).
+template <typename LT>
+__device__ void issue_chunk(const AcceptParams &p, const Item &it, int j, char *stage, uint64_t *full) {
+  constexpr int E = LTraits<LT>::E;
+  const int lane = threadIdx.x & 31;
+  const bool stats = it.kind == WORK_STATS;
+  const int64_t CH = stats ? kStatsChunk : kDrawChunk;
+  const int64_t cv0 = it.v0 + (int64_t)j * CH;
+  const int nv = (int)min(CH, it.v1 - cv0);
+  const bool resid = !stats && it.resid;
+  const LT *row = static_cast<const LT *>(p.logits) + it.R * (int64_t)p.V;
+  const float *qrow = p.draft_probs + (it.D0 + it.i) * (int64_t)p.V;
+  if (p.vec_z && (!resid || p.vec_q)) {
+    if (lane == 0) {
+      const uint32_t zb = (uint32_t)nv * 16u, qb = resid ? (uint32_t)nv * E * 4u : 0u;
+      ptx::mbar_arrive_expect_tx(full, zb + qb);
+      ptx::bulk_load(ptx::smem_u32(stage), row + cv0 * E, zb, full);
+      if (resid) ptx::bulk_load(ptx::smem_u32(stage + kQOffset), qrow + cv0 * E, qb, full);
+    }
+    return;
+  }
+  uint4 *dz = reinterpret_cast<uint4 *>(stage);
+  float *dq = reinterpret_cast<float *>(stage + kQOffset);
+  for (int v = lane; v < nv; v += 32) {
+    dz[v] = load_vec<LT>(row, cv0 + v, p.V, false);
+    if (resid) {
+      float q[E];
+      load_q<E>(qrow, (cv0 + v) * E, p.V, false, q);
+      #pragma unroll
+      for (int i = 0; i < E; ++i) dq[(size_t)v * E + i] = q[i];
+    }
+  }
+  __syncwarp();
+  if (lane == 0) ptx::mbar_arrive(full);
+}
+
+template <typename LT>
+__device__ void producer(const AcceptParams &p, Sm &sm, char *ring) {
+  const int lane = threadIdx.x & 31;
+  long long idle_since = -1;
+  int pend = -1;  // lane 0: a draw ticket taken but not yet usable
+  int n = 0, c = 0;
+  bool ok = true;
+  for (;;) {
+    Item d;
+    int kind = WORK_WAIT;
+    if (lane == 0) kind = pick<LT>(p, sm, d, idle_since, n, pend);
+    kind = __shfl_sync(0xffffffffu, kind, 0);
+    if (kind == WORK_WAIT) {
+      __nanosleep(256);
+      continue;
+    }
+    const int slot = n % kItemSlots;
+    if (!wait_bar(&sm.iq_empty[slot], ((n / kItemSlots) & 1) ^ 1, sm, p)) {
+      ok = false;
+      break;
+    }
+    if (lane == 0) {
+      d.kind = kind;
+      sm.item[slot] = d;
+      ptx::mbar_arrive(&sm.iq_full[slot]);
+    }
+    __syncwarp();
+    if (kind == WORK_EXIT) break;
+    const Item &it = sm.item[slot];
+    for (int j = 0; j < it.nchunks && ok; ++j) {
+      const int stg = c % kStages;
+      if (!wait_bar(&sm.empty[stg], ((c / kStages) & 1) ^ 1, sm, p)) {
+        ok = false;
+        break;
+      }
+      issue_chunk<LT>(p, it, j, ring + (size_t)stg * kStageBytes, &sm.full[stg]);
+      ++c;
+    }
+    if (!ok) break;
+    ++n;
+  }
+  if (!ok) {
+    // given up: let the copies still in flight land before the CTA can exit (bounded)
+    for (int x = c - kStages < 0 ? 0 : c - kStages; x < c; ++x) wait_bar(&sm.full[x % kStages], (x / kStages) & 1, sm, p);
+  }
+}
+
+// ---- the consumers (warps 0..7) -------------------------------------------------------------------
+template <typename LT>
+__device__ void consumers(const AcceptParams &p, Sm &sm, const char *ring, Tab tab) {
+  const bool bf = std::is_same<LT, uint16_t>::value;
+  uint32_t ph = 0;
+  int c = 0;
+  for (int n = 0;; ++n) {
+    const int slot = n % kItemSlots;
+    if (!wait_bar(&sm.iq_full[slot], (n / kItemSlots) & 1, sm, p)) return;
+    Item &it = sm.item[slot];
+    const int kind = it.kind;
+    if (kind != WORK_EXIT && kind != WORK_STATS) {
+      if (threadIdx.x == 0) sm.amb_n = 0;
+      if (bf) ensure_table(it.rec.m, sm, tab, ph, p);
+      cbar(sm, ph, p);
+    }
+    if (kind == WORK_STATS) c_stats<LT>(sm, it, ring, c, ph, p);
+    if (kind == WORK_DRAW) c_draw<LT>(sm, it, bf ? tab : Tab{nullptr, nullptr, nullptr}, ring, c, ph, p);
+    if (kind == WORK_FINISH) c_finish<LT>(sm, it, bf ? tab : Tab{nullptr, nullptr, nullptr}, ring, c, ph, p);
+    cbar(sm, ph, p);  // every consumer is done with the item
+    if (threadIdx.x == 0) ptx::mbar_arrive(&sm.res_ready[slot]);
+    if (kind == WORK_EXIT || vload(sm.abort_)) return;
+  }
+}
+
+}  // namespace
+
+// The acceptance pass (see the file comment): persistent CTAs of consumer, producer and keeper warps.
+template <typename LT>
+__global__ void __launch_bounds__(kCtaThreads, kAcceptCtasPerSM) accept_kernel(const __grid_constant__ AcceptParams p) {
+  extern __shared__ __align__(128) unsigned char s_dyn[];
+  __shared__ Sm sm;
+  char *ring = reinterpret_cast<char *>(s_dyn);
+  const Tab tab{reinterpret_cast<uint32_t *>(s_dyn + kRingBytes),
+                reinterpret_cast<uint32_t *>(s_dyn + kRingBytes + kExpTabSize * sizeof(uint32_t)),
+                reinterpret_cast<float *>(s_dyn + kRingBytes + 2 * kExpTabSize * sizeof(uint32_t))};
+  // launched as a programmatic dependent of the planner: read nothing before it has completed
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const int tid = threadIdx.x, warp = tid >> 5;
+  for (int j = tid; j < 256; j += kCtaThreads) {
+    sm.th[j] = p.tab.hi[j];
+    sm.tl[j] = p.tab.lo[j];
+  }
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      ptx::mbar_init(&sm.full[s], 1);
+      ptx::mbar_init(&sm.empty[s], kCW);
+    }
+    for (int s = 0; s < kItemSlots; ++s) {
+      ptx::mbar_init(&sm.iq_full[s], 1);
+      ptx::mbar_init(&sm.iq_empty[s], 1);
+      ptx::mbar_init(&sm.res_ready[s], 1);
+    }
+    ptx::mbar_init(&sm.cons_bar, kConsumers);
+    ptx::fence_mbar_init();
+    sm.tab_valid = 0;
+    sm.fq_head = sm.fq_tail = 0;
+    sm.keeper_done = 0;
+    sm.abort_ = 0;
+  }
+  __syncthreads();  // the only CTA-wide barrier: set-up
+  if (warp < kCW)
+    consumers<LT>(p, sm, ring, tab);
+  else if (warp == kProducerWarp)
+    producer<LT>(p, sm, ring);
+  else
+    keeper<LT>(p, sm);
 }
 
 // ---- greedy (temperature 0) acceptance -----------------------------------------------------
@@ -921,44 +1728,44 @@ namespace {
 
 template <typename LT>
 cudaError_t set_attr() {
-  // the maximum shared-memory carveout, like the attention kernel, so that these CTAs can share an
-  // SM with an attention CTA when wisp_verify_step runs both at once
-  cudaError_t e = cudaFuncSetAttribute(accept_kernel<LT>, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
+  const int dyn = (int)(kRingBytes + kExpTabBytes);
+  cudaError_t e = cudaFuncSetAttribute(accept_kernel<LT>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(accept_kernel<LT>, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(row_stats_kernel<LT>, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
+    e = cudaFuncSetAttribute(accept_kernel<LT>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
   return e;
 }
 
 template <typename LT>
-cudaError_t stats_t(const AcceptParams &ap, cudaStream_t s) {
-  row_stats_kernel<LT><<<(unsigned)((ap.total_rows * ap.slices + NW - 1) / NW), NT, 0, s>>>(ap);
-  return cudaGetLastError();
-}
-
-template <typename LT>
-cudaError_t walk_t(const AcceptParams &ap, cudaStream_t s) {
-  const int rounds = (ap.vpc + NT - 1) / NT;
+cudaError_t launch_t(const AcceptParams &ap, int sms, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof cfg);
-  cfg.gridDim = dim3((unsigned)((int64_t)ap.B * ap.cluster));
-  cfg.blockDim = dim3(NT);
-  const bool tab = std::is_same<LT, uint16_t>::value && ap.V >= kExpTabMinV;
-  cfg.dynamicSmemBytes = (size_t)rounds * NW * sizeof(ff) + (tab ? kExpTabSize * sizeof(ff) : 0);
+  cfg.gridDim = dim3((unsigned)(sms * kAcceptCtasPerSM));
+  cfg.blockDim = dim3(kCtaThreads);
+  cfg.dynamicSmemBytes = kRingBytes + kExpTabBytes;
   cfg.stream = s;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = (unsigned)ap.cluster;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  // programmatic dependent launch: the clusters may be placed while the previous kernel's last
-  // CTAs run (the kernel waits for it before it reads anything)
-  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[1];
+  // programmatic dependent launch: the CTAs may be placed while the planner runs (the kernel
+  // waits for it before reading anything)
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 2;
+  cfg.numAttrs = pdl ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, accept_kernel<LT>, ap);
+}
+
+// exp(u) for the table's bf16 values, in double (the host's exp) split into two floats.
+void host_exp_table(ff *out) {
+  for (int idx = 0; idx < kExpTabSize; ++idx) {
+    const uint32_t sign = (uint32_t)idx / (kExpTabBinades * 128), rem = (uint32_t)idx % (kExpTabBinades * 128);
+    const uint32_t bits = (sign << 15) | (((rem >> 7) + kExpTabLo) << 7) | (rem & 0x7Fu);
+    const uint32_t f32 = bits << 16;
+    float u;
+    memcpy(&u, &f32, sizeof u);
+    const double v = std::exp((double)u);
+    out[idx].hi = (float)v;
+    out[idx].lo = (float)(v - (double)out[idx].hi);
+  }
 }
 
 }  // namespace
@@ -966,15 +1773,20 @@ cudaError_t walk_t(const AcceptParams &ap, cudaStream_t s) {
 cudaError_t accept_setup() {
   cudaError_t e = set_attr<float>();
   if (e == cudaSuccess) e = set_attr<uint16_t>();
+  if (e == cudaSuccess) {
+    static ff host[kExpTabSize];
+    static bool filled = false;
+    if (!filled) {
+      host_exp_table(host);
+      filled = true;
+    }
+    e = cudaMemcpyToSymbol(g_exp_u, host, sizeof host);
+  }
   return e;
 }
 
-cudaError_t accept_stats_launch(const AcceptParams &p, bool bf16, cudaStream_t s) {
-  return bf16 ? stats_t<uint16_t>(p, s) : stats_t<float>(p, s);
-}
-
-cudaError_t accept_walk_launch(const AcceptParams &p, bool bf16, cudaStream_t s) {
-  return bf16 ? walk_t<uint16_t>(p, s) : walk_t<float>(p, s);
+cudaError_t accept_launch(const AcceptParams &p, bool bf16, int sms, cudaStream_t s, bool pdl) {
+  return bf16 ? launch_t<uint16_t>(p, sms, s, pdl) : launch_t<float>(p, sms, s, pdl);
 }
 
 cudaError_t accept_greedy_launch(const AcceptParams &p, bool bf16, cudaStream_t s) {

@@ -95,6 +95,44 @@ void accept_slices(const wisp_accept_args *c, int sms, int *slices, int *vps) {
   *slices = (int)((nvec + v - 1) / v);
 }
 
+// Work shape of the acceptance kernel: statistics slices per row (enough items, about eight per
+// resident CTA, to balance the persistent CTAs; a slice is a whole number of 4-vector chunks per
+// thread), draw tiles (64 vectors: one warp's share of a draw chunk; no tile records when they
+// would exceed tile_budget bytes) and draw slices per row (about eight per resident CTA over the
+// batch, whole chunks of 256 vectors).
+constexpr size_t kTileBudget = (size_t)256 << 20;
+constexpr size_t kNoAllocTileBudget = (size_t)4 << 20;
+struct AcceptShape {
+  int sslices, svps, dslices, vpd, tile_vecs, ntiles;
+};
+AcceptShape accept_shape(const wisp_accept_args *c, int sms, size_t tile_budget) {
+  const int E = c->logits_dtype == WISP_BF16 ? 8 : 4;
+  const int64_t nvec = ((int64_t)c->V + E - 1) / E;
+  const int64_t ctas = (int64_t)sms * kAcceptCtasPerSM;
+  const int64_t B = c->B > 0 ? c->B : 1;
+  auto cut = [&](int64_t want, int64_t units, int64_t min_vecs, int *n, int *per) {
+    int64_t S = (want + units - 1) / units;
+    const int64_t by_size = (nvec + min_vecs - 1) / min_vecs;
+    if (S > by_size) S = by_size;
+    if (S > 32) S = 32;
+    if (S < 1) S = 1;
+    // whole rounds of the CTA's loads per slice
+    const int64_t v = ((nvec + S - 1) / S + min_vecs - 1) / min_vecs * min_vecs;
+    *per = (int)v;
+    *n = (int)((nvec + v - 1) / v);
+  };
+  AcceptShape sh;
+  cut(8 * ctas, c->total_q_rows > 0 ? c->total_q_rows : 1, (int64_t)kAcceptThreads * kStatsChunkVecs, &sh.sslices,
+      &sh.svps);
+  // a tile is one warp's 64 vectors of a draw chunk; without room for the records, none
+  const int64_t nt = (nvec + 63) / 64;
+  const bool tiles = B * nt * (int64_t)sizeof(TileRec) <= (int64_t)tile_budget;
+  sh.tile_vecs = tiles ? 64 : 0;
+  sh.ntiles = tiles ? (int)nt : 0;
+  cut(8 * ctas, B, kAcceptThreads, &sh.dslices, &sh.vpd);
+  return sh;
+}
+
 // need_probs: the sampling rule reads the draft distributions and the uniforms; the greedy one does not
 wisp_status check_accept(const wisp_accept_args *c, bool need_probs = true) {
   if (!c) return WISP_ERR_INVALID_ARG;
@@ -112,7 +150,7 @@ wisp_status check_accept(const wisp_accept_args *c, bool need_probs = true) {
   return WISP_OK;
 }
 
-Layout make_layout(const wisp_attn_args *a, const wisp_accept_args *c, int sms) {
+Layout make_layout(const wisp_attn_args *a, const wisp_accept_args *c, int sms, size_t tile_budget = kTileBudget) {
   Layout L;
   const int B = a ? a->B : (c ? c->B : 0);
   size_t off = 0;
@@ -141,9 +179,23 @@ Layout make_layout(const wisp_attn_args *a, const wisp_accept_args *c, int sms) 
     L.partials = take(sizeof(float) * (size_t)L.partial_cap);
   }
   if (c && c->B > 0) {
+    const AcceptShape sh = accept_shape(c, sms, tile_budget);
+    const size_t T = (size_t)c->total_q_rows;
+    L.acc_ctr = take(sizeof(AccCounters));
+    L.row_order = take(sizeof(int2) * T);
+    L.row_cnt = take(sizeof(int32_t) * T);
+    L.row_code = take(sizeof(int32_t) * T);
+    L.row_rec = take(sizeof(RowRec) * T);
+    L.sparts = take(sizeof(SlicePart) * T * sh.sslices);
+    L.req_state = take(sizeof(int32_t) * 5 * (size_t)c->B);
+    L.dparts = take(sizeof(DrawPart) * (size_t)c->B * sh.dslices);
+    L.tiles = take(sizeof(TileRec) * ((size_t)c->B * sh.ntiles + 1));
+    // the greedy variant's argmax partials (8 bytes per row and warp slice) share the statistics'
+    // space when they fit, else get their own
     int S = 1, vps = 0;
     accept_slices(c, sms, &S, &vps);
-    L.row_parts = take(sizeof(RowPart) * (size_t)c->total_q_rows * S);
+    const size_t gbytes = 8 * T * S;
+    L.row_parts = gbytes <= sizeof(SlicePart) * T * sh.sslices ? L.sparts : take(gbytes);
   }
   L.total = off;
   return L;
@@ -159,7 +211,8 @@ wisp_status check_ws(void *ws, size_t bytes, const Layout &L) {
   return WISP_OK;
 }
 
-PlanParams plan_params(const wisp_attn_args *a, const wisp_accept_args *c, void *ws, const Layout &L) {
+PlanParams plan_params(const wisp_attn_args *a, const wisp_accept_args *c, void *ws, const Layout &L, int sms,
+                       bool with_accept) {
   PlanParams pp;
   std::memset(&pp, 0, sizeof pp);
   pp.B = a ? a->B : c->B;
@@ -191,6 +244,21 @@ PlanParams plan_params(const wisp_attn_args *a, const wisp_accept_args *c, void 
     pp.order = at<int32_t>(ws, L.order);
   } else {
     pp.Hq = pp.Hkv = 1;
+  }
+  if (c && c->B > 0 && with_accept) {
+    pp.with_accept = 1;
+    pp.sslices = accept_shape(c, sms, kTileBudget).sslices;  // (the statistics slices do not depend on the budget)
+    pp.row_order = at<int2>(ws, L.row_order);
+    pp.row_cnt = at<int32_t>(ws, L.row_cnt);
+    pp.row_code = at<int32_t>(ws, L.row_code);
+    int32_t *rs = at<int32_t>(ws, L.req_state);
+    pp.req_rej = rs;
+    pp.req_claim = rs + c->B;
+    pp.req_dcnt = rs + 3 * (size_t)c->B;
+    pp.queue = rs + 4 * (size_t)c->B;
+    pp.acc_ctr = at<AccCounters>(ws, L.acc_ctr);
+    pp.accepted_len = c->accepted_len;
+    pp.next_token = c->next_token;
   }
   return pp;
 }
@@ -231,7 +299,8 @@ wisp_status launch_attention(const wisp_attn_args *a, void *ws, const Layout &L,
   return attn_combine_launch(ap, bf, s) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
 }
 
-AcceptParams accept_params(const wisp_accept_args *c, void *ws, const Layout &L, int sms) {
+AcceptParams accept_params(const wisp_accept_args *c, void *ws, const Layout &L, int sms,
+                           size_t tile_budget = kTileBudget) {
   AcceptParams ap;
   std::memset(&ap, 0, sizeof ap);
   ap.B = c->B;
@@ -240,9 +309,30 @@ AcceptParams accept_params(const wisp_accept_args *c, void *ws, const Layout &L,
   const size_t esz = bf ? 2 : 4;
   ap.vec_z = ((uintptr_t)c->target_logits % 16 == 0) && ((size_t)c->V * esz % 16 == 0);
   ap.vec_q = c->draft_probs && ((uintptr_t)c->draft_probs % 16 == 0) && ((size_t)c->V * 4 % 16 == 0);
-  accept_slices(c, sms, &ap.slices, &ap.vps);
+  const AcceptShape sh = accept_shape(c, sms, tile_budget);
+  ap.sslices = sh.sslices;
+  ap.svps = sh.svps;
+  ap.dslices = sh.dslices;
+  ap.vpd = sh.vpd;
+  ap.tile_vecs = sh.tile_vecs;
+  ap.ntiles = sh.ntiles;
+  ap.tiles = at<TileRec>(ws, L.tiles);
   ap.total_rows = c->total_q_rows;
-  ap.parts = at<RowPart>(ws, L.row_parts);
+  accept_slices(c, sms, &ap.slices, &ap.vps);
+  ap.parts = at<void>(ws, L.row_parts);
+  ap.row_order = at<int2>(ws, L.row_order);
+  ap.row_cnt = at<int32_t>(ws, L.row_cnt);
+  ap.row_code = at<int32_t>(ws, L.row_code);
+  ap.row_rec = at<RowRec>(ws, L.row_rec);
+  ap.sparts = at<SlicePart>(ws, L.sparts);
+  int32_t *rs = at<int32_t>(ws, L.req_state);
+  ap.req_rej = rs;
+  ap.req_claim = rs + c->B;
+  ap.req_L = rs + 2 * (size_t)c->B;
+  ap.req_dcnt = rs + 3 * (size_t)c->B;
+  ap.queue = rs + 4 * (size_t)c->B;
+  ap.dparts = at<DrawPart>(ws, L.dparts);
+  ap.ctr = at<AccCounters>(ws, L.acc_ctr);
   ap.request_ids = c->request_ids;
   ap.draft_lens = c->draft_lens;
   ap.logits = c->target_logits;
@@ -257,42 +347,35 @@ AcceptParams accept_params(const wisp_accept_args *c, void *ws, const Layout &L,
   ap.req_flag = at<int32_t>(ws, L.req_flag);
   ap.status = at<DeviceStatus>(ws, L.status);
   ap.tab = g_exp2;
-  // one cluster of C CTAs per request: enough CTAs to fill the GPU, each owning a slice of
-  // every row in whole warp tiles (32 vectors of 16 bytes)
-  const int E = bf ? 8 : 4;
-  const int64_t nvec = ((int64_t)c->V + E - 1) / E;
-  const int64_t want = ((int64_t)4 * sms + c->B - 1) / c->B;
-  int64_t C = want < 1 ? 1 : (want > kMaxAcceptCluster ? kMaxAcceptCluster : want);
-  const int64_t max_c = (nvec + 31) / 32;
-  if (C > max_c) C = max_c;
-  ap.cluster = (int)C;
-  ap.vpc = (int)(((nvec + C - 1) / C + 31) / 32 * 32);
   return ap;
 }
 
-wisp_status launch_accept(const wisp_accept_args *c, void *ws, const Layout &L, int sms, cudaStream_t s) {
-  const AcceptParams ap = accept_params(c, ws, L, sms);
-  const bool bf = c->logits_dtype == WISP_BF16;
-  cudaError_t e = accept_stats_launch(ap, bf, s);
-  if (e == cudaSuccess) e = accept_walk_launch(ap, bf, s);
-  return e == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
-}
-
-wisp_status launch_plan(const wisp_attn_args *a, const wisp_accept_args *c, void *ws, const Layout &L,
-                        cudaStream_t s) {
+// with_accept: the planner also lays out the sampling rule's dispatch order and clears its state
+wisp_status launch_plan(const wisp_attn_args *a, const wisp_accept_args *c, void *ws, const Layout &L, int sms,
+                        bool with_accept, cudaStream_t s) {
   if (cudaMemsetAsync(at<DeviceStatus>(ws, L.status), 0, sizeof(DeviceStatus), s) != cudaSuccess)
     return WISP_ERR_CUDA;
-  const PlanParams pp = plan_params(a, c, ws, L);
+  const PlanParams pp = plan_params(a, c, ws, L, sms, with_accept);
   plan_kernel<<<1, 1024, 0, s>>>(pp);
   return cudaGetLastError() == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
 }
 
+// The planner, then the acceptance kernel as its programmatic dependent (its CTAs are placed while
+// the planner runs and wait for it before reading anything).
+wisp_status launch_accept(const wisp_accept_args *c, void *ws, const Layout &L, int sms, cudaStream_t s,
+                          size_t tile_budget = kTileBudget) {
+  wisp_status st = launch_plan(nullptr, c, ws, L, sms, true, s);
+  if (st != WISP_OK || c->B == 0) return st;
+  const AcceptParams ap = accept_params(c, ws, L, sms, tile_budget);
+  return accept_launch(ap, c->logits_dtype == WISP_BF16, sms, s, true) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
+}
+
 }  // namespace
 
-// Workspace of wisp_verify_accept_noalloc: status word, per-request offsets and flags, planner
-// header and the statistics of every logit row.  4 MiB holds them for batches of up to
-// kNoAllocMaxBatch requests and kNoAllocMaxRows logit rows.
-constexpr size_t kNoAllocScratchBytes = 4 << 20;
+// Workspace of wisp_verify_accept_noalloc: status word, per-request offsets, flags and state,
+// planner header, the dispatch order and statistics of every logit row, the draw's slice totals.
+// 16 MiB holds them for batches of up to kNoAllocMaxBatch requests and kNoAllocMaxRows logit rows.
+constexpr size_t kNoAllocScratchBytes = 16 << 20;
 constexpr int kNoAllocMaxBatch = 8192;
 constexpr int kNoAllocMaxRows = 131072;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
@@ -335,7 +418,7 @@ wisp_status wisp_verify_attention(const wisp_attn_args *attn, void *ws, size_t w
   const Layout L = make_layout(attn, nullptr, sms);
   if ((st = check_ws(ws, ws_bytes, L)) != WISP_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if ((st = launch_plan(attn, nullptr, ws, L, s)) != WISP_OK) return st;
+  if ((st = launch_plan(attn, nullptr, ws, L, sms, false, s)) != WISP_OK) return st;
   if (attn->B == 0) return WISP_OK;
   // alone on the stream after the planner: the attention CTAs set up while the planner runs
   return launch_attention(attn, ws, L, s, true);
@@ -348,10 +431,7 @@ wisp_status wisp_verify_accept(const wisp_accept_args *acc, void *ws, size_t ws_
   if ((st = device_setup(&dev, &sms)) != WISP_OK) return st;
   const Layout L = make_layout(nullptr, acc, sms);
   if ((st = check_ws(ws, ws_bytes, L)) != WISP_OK) return st;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if ((st = launch_plan(nullptr, acc, ws, L, s)) != WISP_OK) return st;
-  if (acc->B == 0) return WISP_OK;
-  return launch_accept(acc, ws, L, sms, s);
+  return launch_accept(acc, ws, L, sms, static_cast<cudaStream_t>(stream));
 }
 
 wisp_status wisp_verify_accept_greedy(const wisp_accept_args *acc, void *ws, size_t ws_bytes, void *stream) {
@@ -362,7 +442,7 @@ wisp_status wisp_verify_accept_greedy(const wisp_accept_args *acc, void *ws, siz
   const Layout L = make_layout(nullptr, acc, sms);
   if ((st = check_ws(ws, ws_bytes, L)) != WISP_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if ((st = launch_plan(nullptr, acc, ws, L, s)) != WISP_OK) return st;
+  if ((st = launch_plan(nullptr, acc, ws, L, sms, false, s)) != WISP_OK) return st;
   if (acc->B == 0) return WISP_OK;
   const AcceptParams ap = accept_params(acc, ws, L, sms);
   return accept_greedy_launch(ap, acc->logits_dtype == WISP_BF16, s) == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
@@ -379,24 +459,22 @@ wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args 
   const Layout L = make_layout(attn, acc, sms);
   if ((st = check_ws(ws, ws_bytes, L)) != WISP_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (attn->B == 0) return launch_plan(attn, acc, ws, L, s);
-  // The row statistics of the acceptance pass read only the logits, so they run on the library's
-  // side stream while the planner (one CTA) runs on `s`; the walk and draw follow the attention
-  // on `s` once the statistics are joined back.  (Running the walk concurrently with the
-  // attention was measured to gain nothing: both are issue-bound while active.)
+  if (attn->B == 0) return launch_plan(attn, acc, ws, L, sms, true, s);
+  // One planner for both parts.  The attention follows it on `s` as its programmatic dependent
+  // (persistent, one CTA per SM); the acceptance pass reads only the logits and the planner's
+  // state, so it runs on the library's side stream, forked after the planner and joined back: its
+  // CTAs take the SMs the attention's CTAs leave as they finish.
   DeviceInfo &d = g_dev[dev];
   std::lock_guard<std::mutex> lk(d.step_mu);
+  if ((st = launch_plan(attn, acc, ws, L, sms, true, s)) != WISP_OK) return st;
   const AcceptParams ap = accept_params(acc, ws, L, sms);
   const bool bf = acc->logits_dtype == WISP_BF16;
   bool ok = cudaEventRecord(d.ev_fork, s) == cudaSuccess && cudaStreamWaitEvent(d.side, d.ev_fork, 0) == cudaSuccess;
-  ok = ok && accept_stats_launch(ap, bf, d.side) == cudaSuccess;
+  ok = ok && accept_launch(ap, bf, sms, d.side, false) == cudaSuccess;
   // join what was forked even after a failed launch, so that `s` never runs ahead of `side`
   const bool joined = cudaEventRecord(d.ev_join, d.side) == cudaSuccess;
-  ok = ok && launch_plan(attn, acc, ws, L, s) == WISP_OK;
-  // no programmatic launch here: the row statistics should have the SMs while the planner runs
-  ok = ok && launch_attention(attn, ws, L, s, false) == WISP_OK;
+  ok = ok && launch_attention(attn, ws, L, s, true) == WISP_OK;
   const bool waited = joined && cudaStreamWaitEvent(s, d.ev_join, 0) == cudaSuccess;
-  ok = ok && waited && accept_walk_launch(ap, bf, s) == cudaSuccess;
   return ok && waited ? WISP_OK : WISP_ERR_CUDA;
 }
 
@@ -423,15 +501,13 @@ wisp_status wisp_verify_accept_noalloc(const wisp_accept_args *acc, void *stream
   if (acc->B > kNoAllocMaxBatch || acc->total_q_rows > kNoAllocMaxRows) return WISP_ERR_UNSUPPORTED;
   int dev = 0, sms = 0;
   if ((st = device_setup(&dev, &sms)) != WISP_OK) return st;
-  const Layout L = make_layout(nullptr, acc, sms);
+  const Layout L = make_layout(nullptr, acc, sms, kNoAllocTileBudget);
   if (L.total > kNoAllocScratchBytes) return WISP_ERR_UNSUPPORTED;
   void *ws = nullptr;
   if ((st = noalloc_scratch(dev, &ws)) != WISP_OK) return st;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // the planner clears the status word (the only field that must start at zero) on `s` first
-  if ((st = launch_plan(nullptr, acc, ws, L, s)) != WISP_OK) return st;
-  if (acc->B == 0) return WISP_OK;
-  return launch_accept(acc, ws, L, sms, s);
+  // the planner clears the status word and the launch's counters and per-row / per-request state
+  // (everything that must start at zero) on `stream` first
+  return launch_accept(acc, ws, L, sms, static_cast<cudaStream_t>(stream), kNoAllocTileBudget);
 }
 
 const char *wisp_verify_status_string(wisp_status s) {

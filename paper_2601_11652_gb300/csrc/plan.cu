@@ -44,6 +44,93 @@ __device__ int64_t block_scan(int64_t v, int64_t *s_warp, int64_t *total) {
   return res;
 }
 
+// The acceptance pass's dispatch order and state.  Rows are listed level-major: row index 0 of
+// every valid request, then row index 1, ... (the requests of a level in decreasing draft length, so
+// that request r holds the same position pos(r) in every level it reaches).  The decision of row i
+// of a request is then usually known before its row i + 1 comes up, and the acceptance kernel skips
+// rows past a rejection.  Also clears the per-row and per-request state of the launch and gives the
+// requests this planner refused -1 outputs.
+__device__ void plan_accept(const PlanParams &p, int64_t *s_warp) {
+  constexpr int KB = kMaxDraft + 1;  // draft lengths 0..kMaxDraft
+  __shared__ int32_t s_n[KB + 1];    // level sizes n_i = #{valid r : k_r >= i}, then cursors
+  __shared__ int32_t s_ls[KB + 1];   // level starts
+  const int tid = threadIdx.x;
+  __syncthreads();  // pass 1's flags and offsets are visible to every thread
+  for (int b = tid; b <= KB; b += kThreads) s_n[b] = 0;
+  __syncthreads();
+  int nv = 0;
+  for (int r = tid; r < p.B; r += kThreads) {
+    p.req_rej[r] = INT32_MAX;
+    p.req_claim[r] = 0;
+    p.req_dcnt[r] = 0;
+    p.queue[r] = -1;
+    if (p.req_flag[r] == REQ_OK) {
+      atomicAdd(&s_n[p.draft_lens[r]], 1);  // histogram of k
+      ++nv;
+    } else {
+      p.accepted_len[r] = -1;
+      p.next_token[r] = -1;
+    }
+  }
+  for (int64_t j = tid; j < p.total_q_rows; j += kThreads) {
+    p.row_cnt[j] = 0;
+    p.row_code[j] = 0;
+  }
+  int64_t nvalid;
+  (void)block_scan(nv, s_warp, &nvalid);
+  // n_i: suffix sums of the histogram (buckets in decreasing order, in chunks of kThreads)
+  int64_t carry = 0;
+  for (int base = 0; base < KB; base += kThreads) {
+    const int b = KB - 1 - (base + tid);
+    const int64_t c = b >= 0 ? s_n[b] : 0;
+    int64_t tot;
+    const int64_t incl = block_scan(c, s_warp, &tot);
+    if (b >= 0) s_n[b] = (int32_t)(carry + incl);
+    carry += tot;
+    __syncthreads();
+  }
+  if (tid == 0) s_n[KB] = 0;
+  __syncthreads();
+  // level starts: exclusive prefix sums of n_i
+  carry = 0;
+  for (int base = 0; base <= KB; base += kThreads) {
+    const int b = base + tid;
+    const int64_t c = b <= KB ? s_n[b] : 0;
+    int64_t tot;
+    const int64_t incl = block_scan(c, s_warp, &tot);
+    if (b <= KB) s_ls[b] = (int32_t)(carry + incl - c);
+    carry += tot;
+  }
+  __syncthreads();
+  const int64_t rows_valid = carry;
+  // cursors: in every level, the requests with a larger k come first; bucket k starts at n_{k+1}
+  int32_t nxt[2];
+  for (int j = 0; j < 2; ++j) {
+    const int b = j * kThreads + tid;
+    nxt[j] = b < KB ? s_n[b + 1] : 0;
+  }
+  __syncthreads();
+  for (int j = 0; j < 2; ++j) {
+    const int b = j * kThreads + tid;
+    if (b < KB) s_n[b] = nxt[j];
+  }
+  __syncthreads();
+  for (int r = tid; r < p.B; r += kThreads) {
+    if (p.req_flag[r] != REQ_OK) continue;
+    const int k = p.draft_lens[r];
+    const int pos = atomicAdd(&s_n[k], 1);
+    for (int i = 0; i <= k; ++i) p.row_order[s_ls[i] + pos] = make_int2(r, i);
+  }
+  if (tid == 0) {
+    p.acc_ctr->n_items = (int32_t)(rows_valid * p.sslices);
+    p.acc_ctr->n_valid = (int32_t)nvalid;
+    p.acc_ctr->q_reserve = 0;
+    p.acc_ctr->q_head = 0;
+    p.acc_ctr->n_claimed = 0;
+    p.acc_ctr->stats_next = 0;
+  }
+}
+
 }  // namespace
 
 __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
@@ -102,6 +189,7 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
       atomicCAS(&p.status->code, 0, (int32_t)WISP_DEV_BAD_LENGTH);
     }
   }
+  if (p.with_accept) plan_accept(p, s_warp);
   if (!p.with_attention) return;
   __syncthreads();
 

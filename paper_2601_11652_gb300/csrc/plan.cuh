@@ -33,6 +33,23 @@ constexpr int kItemsPerSM = 2;     // work items per SM when (request, head) pai
 constexpr int kMinChunk = 256;     // never split a sequence below this many tokens
 constexpr int kChunkAlign = 128;   // chunk starts are multiples of the KV tile
 
+// Global counters of one acceptance launch (zeroed by the planner).
+struct AccCounters {
+  int32_t n_items;       // statistics items (slices x rows of valid requests)
+  int32_t n_valid;       // requests the planner accepted
+  int32_t pad0[30];
+  // draw queue: requests pushed, and draw tickets taken (ticket = queue entry * draw slices +
+  // slice), each on its own 128-byte line
+  int32_t q_reserve;
+  int32_t pad1[31];
+  int32_t q_head;
+  int32_t pad4[31];
+  int32_t n_claimed;     // requests whose L is known (queued) or that failed
+  int32_t pad2[31];
+  int32_t stats_next;    // next statistics item to claim (its own line)
+  int32_t pad3[31];
+};
+
 // Byte offsets of every region inside the caller's workspace.
 struct Layout {
   size_t status = 0;          // DeviceStatus (256 B)
@@ -46,7 +63,18 @@ struct Layout {
   size_t items = 0;           // WorkItem [max_items]
   size_t order = 0;           // int32 [max_items]  dispatch order of the items (largest first)
   size_t partials = 0;        // float [partial_cap]
-  size_t row_parts = 0;       // RowPart [total_q_rows, slices] statistics of the logit rows
+  // acceptance pass (sampling rule)
+  size_t acc_ctr = 0;         // AccCounters
+  size_t row_order = 0;       // int2 [total_q_rows] (request, row index), level-major
+  size_t row_cnt = 0;         // int32 [total_q_rows]
+  size_t row_code = 0;        // int32 [total_q_rows]
+  size_t row_rec = 0;         // RowRec [total_q_rows]
+  size_t sparts = 0;          // SlicePart [total_q_rows, sslices]
+  size_t req_state = 0;       // int32 [5, B]: lowest rejecting row, claim, L, finished draw slices, queue
+  size_t dparts = 0;          // DrawPart [B, dslices]
+  size_t tiles = 0;           // TileRec [B, ntiles]
+  // greedy variant
+  size_t row_parts = 0;       // argmax partials [total_q_rows, slices]
   size_t total = 0;
   int64_t max_items = 0;
   int64_t partial_cap = 0;    // floats
@@ -68,6 +96,14 @@ struct PlanParams {
   int32_t *req_item_begin, *req_chunks, *pair_done;
   WorkItem *items;
   int32_t *order;
+  // acceptance pass: level-major dispatch order of the logit rows and the launch's state
+  int with_accept;
+  int sslices;                 // statistics slices per row
+  int2 *row_order;
+  int32_t *row_cnt, *row_code;
+  int32_t *req_rej, *req_claim, *req_dcnt, *queue;
+  AccCounters *acc_ctr;
+  int32_t *accepted_len, *next_token;  // -1 for the requests the planner refuses
 };
 
 __global__ void plan_kernel(const PlanParams p);
