@@ -437,12 +437,11 @@ struct FinTask {
   double thr, Zu;
 };
 
-// The draw's per-CTA exp table (dynamic shared memory): the fixed-point value as two 32-bit words
-// and the float value, three arrays of 4-byte entries (random 4-byte loads cost far less than
-// random 8-byte ones).
+// The draw's per-CTA exp table (dynamic shared memory): the fixed-point value as two 32-bit words,
+// two arrays of 4-byte entries (random 4-byte loads cost far less than random 8-byte ones); hi
+// follows lo directly.
 struct Tab {
   uint32_t *lo, *hi;
-  float *f;
 };
 
 struct Sm {
@@ -458,6 +457,7 @@ struct Sm {
   double dred[kCW];
   unsigned tab_m_bits;
   int tab_valid;
+  int tab_mode;
   int amb_n;
   AmbElem amb[kAmbPerSlice];
   int first, lastpos;
@@ -496,42 +496,76 @@ __device__ __forceinline__ void cbar(Sm &sm, uint32_t &ph, const AcceptParams &p
   ++ph;
 }
 
-// Build the per-CTA table of round(2^56 exp(u - m)) over the table's bf16 values u (0 for u > m),
-// unless it already holds this m: from exp(u) exp(-m) when -m is itself a table value, else
-// directly; both in double-float.  Called by every consumer thread.
+// The consumers' exp table (Tab) holds round(2^56 exp(u - m)) for the item's row maximum m:
+// nothing to do when it already does.  Else from the launch's global copy for this m when one is
+// ready (any CTA's draw of a row with the same maximum wrote it), or built here, from
+// exp(u) exp(-m) when -m is itself a table value, else directly, both in double-float, and then
+// published when the slot for m is free.  Called by every consumer thread.
 __device__ void ensure_table(float m, Sm &sm, Tab tab, uint32_t &ph, const AcceptParams &p) {
   constexpr int PER = (kExpTabSize + kConsumers - 1) / kConsumers;
+  constexpr int NW4 = (int)(kExpTabBytes / 16);  // 16-byte words of a table
   const unsigned mb = __float_as_uint(m);
   if (sm.tab_valid && sm.tab_m_bits == mb) return;
-  cbar(sm, ph, p);  // no consumer still reads the previous table
-  const int mi = exp_tab_index((mb >> 16) ^ 0x8000u);  // -m (m is a bf16 value)
-  if (mi >= 0) {
-    const ff Em = g_exp_u[mi];
-    ff g[PER];  // every load first: one round trip
+  const int slot = (int)((mb >> 16) & (kTabCacheSlots - 1));
+  uint4 *gt = p.tcache ? reinterpret_cast<uint4 *>(p.tcache + (size_t)slot * 2 * kExpTabSize) : nullptr;
+  if (threadIdx.x == 0) {
+    int mode = 0;  // 0 build, 1 build and publish, 2 copy the published table
+    if (gt) {
+      const int st = ptx::ld_acquire_gpu(&p.ctr->tab_state[slot]);
+      if (st == 2 && ld_vol((const int32_t *)&p.ctr->tab_m[slot]) == (int32_t)mb)
+        mode = 2;
+      else if (st == 0 && atomicCAS(&p.ctr->tab_state[slot], 0, 1) == 0)
+        mode = 1;
+    }
+    sm.tab_mode = mode;
+  }
+  cbar(sm, ph, p);  // no consumer still reads the previous table; the mode is visible
+  const int mode = vload(sm.tab_mode);
+  uint4 *st4 = reinterpret_cast<uint4 *>(tab.lo);  // lo and hi are contiguous
+  if (mode == 2) {
+    uint4 g[(NW4 + kConsumers - 1) / kConsumers];
 #pragma unroll
-    for (int j = 0; j < PER; ++j) {
-      const int idx = threadIdx.x + j * kConsumers;
-      g[j] = idx < kExpTabSize ? g_exp_u[idx] : ff{0.0f, 0.0f};
+    for (int j = 0; j < (NW4 + kConsumers - 1) / kConsumers; ++j) {
+      const int x = threadIdx.x + j * kConsumers;
+      if (x < NW4) g[j] = __ldcg(gt + x);
     }
 #pragma unroll
-    for (int j = 0; j < PER; ++j) {
-      const int idx = threadIdx.x + j * kConsumers;
-      if (idx < kExpTabSize) {
-        const bool used = bf16_bits_to_float(exp_tab_bits(idx)) <= m;
-        const ff e = ff_mul(g[j], Em);
-        const unsigned long long fx = used ? ff_to_fix(e) : 0ull;
-        tab.lo[idx] = (uint32_t)fx;
-        tab.hi[idx] = (uint32_t)(fx >> 32);
-        tab.f[idx] = used ? e.hi : 0.0f;
-      }
+    for (int j = 0; j < (NW4 + kConsumers - 1) / kConsumers; ++j) {
+      const int x = threadIdx.x + j * kConsumers;
+      if (x < NW4) st4[x] = g[j];
     }
   } else {
-    for (int idx = threadIdx.x; idx < kExpTabSize; idx += kConsumers) {
-      const float u = bf16_bits_to_float(exp_tab_bits(idx));
-      const Wt v = u <= m ? exp_fix_direct(u, m, sm.th, sm.tl) : Wt{0, 0.0f};
-      tab.lo[idx] = (uint32_t)v.fix;
-      tab.hi[idx] = (uint32_t)(v.fix >> 32);
-      tab.f[idx] = v.f;
+    const int mi = exp_tab_index((mb >> 16) ^ 0x8000u);  // -m (m is a bf16 value)
+    if (mi >= 0) {
+      const ff Em = g_exp_u[mi];
+      ff g[PER];  // every load first: one round trip
+#pragma unroll
+      for (int j = 0; j < PER; ++j) {
+        const int idx = threadIdx.x + j * kConsumers;
+        g[j] = idx < kExpTabSize ? g_exp_u[idx] : ff{0.0f, 0.0f};
+      }
+#pragma unroll
+      for (int j = 0; j < PER; ++j) {
+        const int idx = threadIdx.x + j * kConsumers;
+        if (idx < kExpTabSize) {
+          const bool used = bf16_bits_to_float(exp_tab_bits(idx)) <= m;
+          const unsigned long long fx = used ? ff_to_fix(ff_mul(g[j], Em)) : 0ull;
+          tab.lo[idx] = (uint32_t)fx;
+          tab.hi[idx] = (uint32_t)(fx >> 32);
+        }
+      }
+    } else {
+      for (int idx = threadIdx.x; idx < kExpTabSize; idx += kConsumers) {
+        const float u = bf16_bits_to_float(exp_tab_bits(idx));
+        const unsigned long long fx = u <= m ? exp_fix_direct(u, m, sm.th, sm.tl).fix : 0ull;
+        tab.lo[idx] = (uint32_t)fx;
+        tab.hi[idx] = (uint32_t)(fx >> 32);
+      }
+    }
+    if (mode == 1) {
+      cbar(sm, ph, p);  // the whole table is in shared memory
+      for (int x = threadIdx.x; x < NW4; x += kConsumers) __stcg(gt + x, st4[x]);
+      __threadfence();
     }
   }
   if (threadIdx.x == 0) {
@@ -539,17 +573,23 @@ __device__ void ensure_table(float m, Sm &sm, Tab tab, uint32_t &ph, const Accep
     sm.tab_valid = 1;
   }
   cbar(sm, ph, p);
+  if (mode == 1 && threadIdx.x == 0) {
+    // every consumer's part of the copy is fenced and behind the barrier: publish it
+    st_vol((int32_t *)&p.ctr->tab_m[slot], (int32_t)mb);
+    __threadfence();
+    ptx::st_release_gpu(&p.ctr->tab_state[slot], 2);
+  }
 }
 
-// The E weights of one vector: round(2^56 exp(z - m)) and exp(z - m) as a float.  From the table for
-// bf16 values in its range (almost every logit); the others (|z| < 2^-8, |z| >= 64, +-0, a table
-// not given) directly, entered once per vector that needs it.
+// The E weights of one vector: round(2^56 exp(z - m)).  From the table for bf16 values in its
+// range (almost every logit); the others (|z| < 2^-16, |z| >= 64, +-0, a table not given) directly,
+// entered once per vector that needs it.
 template <typename LT>
 __device__ __forceinline__ void weights(const uint4 &w, float m, const Sm &sm, Tab tab,
-                                        unsigned long long (&fx)[LTraits<LT>::E], float (&fl)[LTraits<LT>::E]);
+                                        unsigned long long (&fx)[LTraits<LT>::E]);
 template <>
 __device__ __forceinline__ void weights<uint16_t>(const uint4 &w, float m, const Sm &sm, Tab tab,
-                                                  unsigned long long (&fx)[8], float (&fl)[8]) {
+                                                  unsigned long long (&fx)[8]) {
   bool slow = false;
   int idx[8];
 #pragma unroll
@@ -561,37 +601,28 @@ __device__ __forceinline__ void weights<uint16_t>(const uint4 &w, float m, const
     slow |= idx[i] == -1;
   }
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
+  for (int i = 0; i < 8; ++i)
     fx[i] = idx[i] >= 0 ? ((unsigned long long)tab.hi[idx[i]] << 32) | tab.lo[idx[i]] : 0ull;
-    fl[i] = idx[i] >= 0 ? tab.f[idx[i]] : 0.0f;
-  }
   if (slow) {
     #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      if (idx[i] == -1) {
-        const Wt e = exp_fix_direct(vec_elem<uint16_t>(w, i), m, sm.th, sm.tl);
-        fx[i] = e.fix;
-        fl[i] = e.f;
-      }
-    }
+    for (int i = 0; i < 8; ++i)
+      if (idx[i] == -1) fx[i] = exp_fix_direct(vec_elem<uint16_t>(w, i), m, sm.th, sm.tl).fix;
   }
 }
 template <>
 __device__ __forceinline__ void weights<float>(const uint4 &w, float m, const Sm &sm, Tab,
-                                               unsigned long long (&fx)[4], float (&fl)[4]) {
+                                               unsigned long long (&fx)[4]) {
   #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const Wt e = exp_fix_direct(vec_elem<float>(w, i), m, sm.th, sm.tl);
-    fx[i] = e.fix;
-    fl[i] = e.f;
-  }
+  for (int i = 0; i < 4; ++i) fx[i] = exp_fix_direct(vec_elem<float>(w, i), m, sm.th, sm.tl).fix;
+}
+
+// A fixed-point weight (units 2^-56, at most 2^56) as a float, within 2^-23 of its value relative:
+// the high word converts exactly, the low one with one rounding, and one rounding in the sum.
+__device__ __forceinline__ float fix_to_float(unsigned long long x) {
+  return __fmaf_rn(__uint2float_rn((uint32_t)(x >> 32)), 0x1p-24f, __uint2float_rn((uint32_t)x) * 0x1p-56f);
 }
 
 __device__ __forceinline__ double ff_to_double_(ff a) { return (double)a.hi + (double)a.lo; }
-__device__ __forceinline__ ff ff_warp_sum(ff a) {
-  for (int o = 16; o > 0; o >>= 1) a = ff_add(a, ff_shfl_xor(a, o));
-  return a;
-}
 
 // Draw weight of one element in units of 2^-56, in double: the residual max(0, e - q Z) (Z = Zu in
 // the same units) or e itself.  fmax drops a NaN q (no mass), as max(0, p - q) does.
@@ -606,8 +637,7 @@ __device__ __forceinline__ double vec_weight(const uint4 &w, const float *q, boo
                                              const Sm &sm, Tab tab) {
   constexpr int E = LTraits<LT>::E;
   unsigned long long fx[E];
-  float fl[E];
-  weights<LT>(w, m, sm, tab, fx, fl);
+  weights<LT>(w, m, sm, tab, fx);
   const float Zf = (float)(Zu * 0x1p-56);
   const float zh = Zf * (1.0f + 0x1p-20f), zl = Zf * (1.0f - 0x1p-20f);
   unsigned long long sp = 0;
@@ -617,10 +647,10 @@ __device__ __forceinline__ double vec_weight(const uint4 &w, const float *q, boo
   for (int i = 0; i < E; ++i) {
     if (!residual) {
       sp += fx[i];
-    } else if (q[i] >= 0.0f && fl[i] > q[i] * zh) {
+    } else if (q[i] >= 0.0f && fix_to_float(fx[i]) > q[i] * zh) {
       sp += fx[i];
       ff_acc(sq, q[i]);
-    } else if (fl[i] > q[i] * zl) {
+    } else if (fix_to_float(fx[i]) > q[i] * zl) {
       ad += weight_d(fx[i], q[i], true, Zu);
     }
   }
@@ -676,17 +706,16 @@ __device__ void c_stats(Sm &sm, Item &it, const char *ring, int &c, uint32_t &ph
   }
 }
 
-// Warp sum of one 64-bit value per lane as a U96 (the 32-bit halves summed separately).
-__device__ __forceinline__ U96 warp_sum_u64(unsigned long long x) {
-  unsigned long long lo = x & 0xFFFFFFFFull, hi = x >> 32;
-  for (int o = 16; o > 0; o >>= 1) {
-    lo += __shfl_xor_sync(0xffffffffu, lo, o);
-    hi += __shfl_xor_sync(0xffffffffu, hi, o);
-  }
+// Warp sum of one value x <= 2^61 per lane as a U96: three 32-bit warp reductions of the 27-bit
+// fields of x (each field sum is below 2^32), recombined.
+__device__ __forceinline__ U96 warp_sum_u61(unsigned long long x) {
+  const unsigned a = __reduce_add_sync(0xffffffffu, (unsigned)(x & 0x7FFFFFFu));
+  const unsigned b = __reduce_add_sync(0xffffffffu, (unsigned)((x >> 27) & 0x7FFFFFFu));
+  const unsigned c = __reduce_add_sync(0xffffffffu, (unsigned)(x >> 54));  // < 2^13
   U96 r = u96_zero();
-  r.lo = lo;
-  u96_add(r, hi << 32);
-  r.hi += (unsigned)(hi >> 32);
+  r.lo = (unsigned long long)a + ((unsigned long long)b << 27);  // < 2^60
+  r.hi = c >> 10;
+  u96_add(r, (unsigned long long)(c & 0x3FFu) << 54);
   return r;
 }
 // Warp sum of non-negative double-float values (same-sign addition: no cancellation).
@@ -763,28 +792,27 @@ __device__ void c_draw(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint
     for (int h = 0; h < 2; ++h) {
       if (!have[h]) continue;
       unsigned long long fx[E];
-      float fl[E];
-      weights<LT>(w[h], rec.m, sm, tab, fx, fl);
+      weights<LT>(w[h], rec.m, sm, tab, fx);
       bool amb = false;
 #pragma unroll
       for (int i = 0; i < E; ++i) {
         sa += fx[i];
         if (residual) {
-          const float qi = q[h][i];
-          const bool pos = qi >= 0.0f && fl[i] > qi * zhi;
+          const float qi = q[h][i], fl = fix_to_float(fx[i]);
+          const bool pos = qi >= 0.0f && fl > qi * zhi;
           if (pos) sp += fx[i];
           if (i & 1)
             ff_acc(tq2, pos ? qi : 0.0f);
           else
             ff_acc(tq, pos ? qi : 0.0f);
-          amb |= !pos && fl[i] > qi * zlo;  // neither certainly positive nor certainly without mass
+          amb |= !pos && fl > qi * zlo;  // neither certainly positive nor certainly without mass
         }
       }
       if (amb) {
         #pragma unroll
         for (int i = 0; i < E; ++i) {
-          const float qi = q[h][i];
-          if (!(qi >= 0.0f && fl[i] > qi * zhi) && fl[i] > qi * zlo) {
+          const float qi = q[h][i], fl = fix_to_float(fx[i]);
+          if (!(qi >= 0.0f && fl > qi * zhi) && fl > qi * zlo) {
             const int a = atomicAdd(&sm.amb_n, 1);
             if (a < kAmbPerSlice) {
               sm.amb[a].e = fx[i];
@@ -797,12 +825,15 @@ __device__ void c_draw(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint
     }
     if (residual) tq = ff_add_pos(tq, tq2);
     // the warp's tile: its sums, warp-wide, into the tile records
-    const U96 A_ = warp_sum_u64(sa), P_ = residual ? warp_sum_u64(sp) : u96_zero();
+    // per lane at most 16 weights of at most 2^56 each
+    const U96 A_ = warp_sum_u61(sa), P_ = residual ? warp_sum_u61(sp) : u96_zero();
     const ff Q_ = residual ? ff_warp_sum_pos(tq) : ff{0.0f, 0.0f};
     if (p.tile_vecs && lane == 0 && cv0 + wi * TV < it.v1) {
       TileRec r;
-      r.e_all = u96_to_double(A_);
-      r.e_p = u96_to_double(P_);
+      r.a_lo = A_.lo;
+      r.a_hi = A_.hi;
+      r.p_lo = P_.lo;
+      r.p_hi = P_.hi;
       r.q_hi = Q_.hi;
       r.q_lo = Q_.lo;
       trec[(cv0 + wi * TV) / TV] = r;
@@ -900,8 +931,7 @@ __device__ void c_finish(Sm &sm, Item &it, Tab tab, const char *ring, int &c, ui
       if (tid == sm.first) {
         // this thread's elements in order, with exact weights
         unsigned long long fx[E];
-        float fl[E];
-        weights<LT>(w, it.rec.m, sm, tab, fx, fl);
+        weights<LT>(w, it.rec.m, sm, tab, fx);
         const double r2 = thr - (incl - wv);
         double acc = 0.0;
         int tok = -1, lastv = -1;
@@ -938,8 +968,7 @@ __device__ void c_finish(Sm &sm, Item &it, Tab tab, const char *ring, int &c, ui
       for (int i = 0; i < E; ++i) q[i] = 0.0f;
       if (residual) load_q<E>(qrow, last_vec * E, p.V, p.vec_q != 0, q);
       unsigned long long fx[E];
-      float fl[E];
-      weights<LT>(w, it.rec.m, sm, tab, fx, fl);
+      weights<LT>(w, it.rec.m, sm, tab, fx);
       #pragma unroll
       for (int i = 0; i < E; ++i) {
         const int64_t v = last_vec * E + i;
@@ -1046,7 +1075,7 @@ __device__ double warp_range_weight(const AcceptParams &p, const Sm &sm, const L
     #pragma unroll
     for (int i = 0; i < E; ++i) q[i] = 0.0f;
     if (qrow) load_q<E>(qrow, vi * E, p.V, p.vec_q != 0, q);
-    acc += vec_weight<LT>(w, q, qrow != nullptr, m, Zu, sm, Tab{nullptr, nullptr, nullptr});
+    acc += vec_weight<LT>(w, q, qrow != nullptr, m, Zu, sm, Tab{nullptr, nullptr});
   }
   for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
   return acc;
@@ -1122,6 +1151,14 @@ __device__ void k_stats(const AcceptParams &p, Sm &sm, const Item &it) {
 }
 
 // Post a finish task to this CTA's producer (bounded wait for room).
+// One of a tile record's integer sums (over the elements with p > q when pos, else all).
+__device__ __forceinline__ U96 tile_u96(const TileRec *t, bool pos) {
+  U96 r = u96_zero();
+  r.lo = __ldcg(pos ? &t->p_lo : &t->a_lo);
+  r.hi = __ldcg(pos ? &t->p_hi : &t->a_hi);
+  return r;
+}
+
 __device__ bool post_finish(Sm &sm, const FinTask &f, const AcceptParams &p) {
   const long long t0 = clock64();
   while (vload(sm.fq_tail) - vload(sm.fq_head) >= kFinQ) {
@@ -1266,13 +1303,13 @@ __device__ void k_draw(const AcceptParams &p, Sm &sm, const Item &it) {
       if (d_over) {
         w = 0.0;  // filled below, one tile at a time, by the whole warp
       } else if (resid) {
-        w = __ldcg(&tr[t].e_p) - Zu * ((double)__ldcg(&tr[t].q_hi) + (double)__ldcg(&tr[t].q_lo));
+        w = u96_to_double(tile_u96(tr + t, true)) - Zu * ((double)__ldcg(&tr[t].q_hi) + (double)__ldcg(&tr[t].q_lo));
         for (int j = 0; j < nad; ++j) {
           const int64_t vt = (int64_t)(__ldcg(&dd->amb[j].v) / E) / p.tile_vecs;
           if (vt == t) w += weight_d(__ldcg(&dd->amb[j].e), __ldcg(&dd->amb[j].q), true, Zu);
         }
       } else {
-        w = __ldcg(&tr[t].e_all);
+        w = u96_to_double(tile_u96(tr + t, false));
       }
     }
     if (d_over) {
@@ -1563,8 +1600,8 @@ __device__ void consumers(const AcceptParams &p, Sm &sm, const char *ring, Tab t
       cbar(sm, ph, p);
     }
     if (kind == WORK_STATS) c_stats<LT>(sm, it, ring, c, ph, p);
-    if (kind == WORK_DRAW) c_draw<LT>(sm, it, bf ? tab : Tab{nullptr, nullptr, nullptr}, ring, c, ph, p);
-    if (kind == WORK_FINISH) c_finish<LT>(sm, it, bf ? tab : Tab{nullptr, nullptr, nullptr}, ring, c, ph, p);
+    if (kind == WORK_DRAW) c_draw<LT>(sm, it, bf ? tab : Tab{nullptr, nullptr}, ring, c, ph, p);
+    if (kind == WORK_FINISH) c_finish<LT>(sm, it, bf ? tab : Tab{nullptr, nullptr}, ring, c, ph, p);
     cbar(sm, ph, p);  // every consumer is done with the item
     if (threadIdx.x == 0) ptx::mbar_arrive(&sm.res_ready[slot]);
     if (kind == WORK_EXIT || vload(sm.abort_)) return;
@@ -1580,8 +1617,7 @@ __global__ void __launch_bounds__(kCtaThreads, kAcceptCtasPerSM) accept_kernel(c
   __shared__ Sm sm;
   char *ring = reinterpret_cast<char *>(s_dyn);
   const Tab tab{reinterpret_cast<uint32_t *>(s_dyn + kRingBytes),
-                reinterpret_cast<uint32_t *>(s_dyn + kRingBytes + kExpTabSize * sizeof(uint32_t)),
-                reinterpret_cast<float *>(s_dyn + kRingBytes + 2 * kExpTabSize * sizeof(uint32_t))};
+                reinterpret_cast<uint32_t *>(s_dyn + kRingBytes + kExpTabSize * sizeof(uint32_t))};
   // launched as a programmatic dependent of the planner: read nothing before it has completed
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int tid = threadIdx.x, warp = tid >> 5;

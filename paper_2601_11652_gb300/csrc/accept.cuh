@@ -8,15 +8,15 @@ namespace wisp {
 constexpr int kAcceptThreads = 256;  // consumer threads of an acceptance CTA (8 warps; plus a producer and a keeper warp)
 constexpr int kAcceptCtasPerSM = 2;  // resident CTAs per SM of the persistent acceptance kernel
 constexpr int kStatsChunkVecs = 3;   // 16-byte vectors per consumer thread in one chunk of the statistics stream
-constexpr int kAmbPerSlice = 8;
-constexpr int kMaxSlices = 32;       // warp slices per row of the greedy variant      // residual elements per draw slice whose sign is left to the finisher
+constexpr int kAmbPerSlice = 8;      // residual elements per draw slice whose sign is left to the finisher
+constexpr int kMaxSlices = 32;       // warp slices per row of the greedy variant
 
-// Per-CTA table of exp(u - m) for the bf16 values u with 2^-8 <= |u| < 2^6 (exponent fields
+// Per-CTA table of exp(u - m) for the bf16 values u with 2^-16 <= |u| < 2^6 (exponent fields
 // kExpTabLo .. kExpTabLo + kExpTabBinades - 1, both signs): 64-bit fixed-point values of the draw.
-constexpr int kExpTabLo = 119;
-constexpr int kExpTabBinades = 14;
+constexpr int kExpTabLo = 111;
+constexpr int kExpTabBinades = 22;
 constexpr int kExpTabSize = 2 * kExpTabBinades * 128;
-constexpr size_t kExpTabBytes = kExpTabSize * 3 * sizeof(uint32_t);  // fixed point (two words) + float
+constexpr size_t kExpTabBytes = kExpTabSize * 2 * sizeof(uint32_t);  // fixed point, two 32-bit words
 // Fixed-point scale of the draw's weights: exp(z - m) in [0, 1] is held as round(2^56 exp(z - m)),
 // so that a thread sums up to 2^7 of them in 64 bits and every sum is exact and order-free.
 constexpr int kFixShift = 56;
@@ -70,10 +70,12 @@ struct DrawPart {
 };
 
 // Sums of one tile (tile_vecs consecutive vectors of row L) written by the draw: over all elements
-// and over the elements with p > q (certainly) of exp(z - m) in units of 2^-56, and of q over the
-// latter (double-float).  The finisher locates the crossing tile from them.
+// and over the elements with p > q (certainly) of exp(z - m) in units of 2^-56 (96-bit integers:
+// low 64 bits, high 32 bits), and of q over the latter (double-float).  The crossing search
+// locates the tile from them.
 struct TileRec {
-  double e_all, e_p;
+  unsigned long long a_lo, p_lo;
+  unsigned int a_hi, p_hi;
   float q_hi, q_lo;
 };
 
@@ -103,6 +105,7 @@ struct AcceptParams {
   int32_t *queue;          // [B] requests ready to draw (-1: not yet written)
   DrawPart *dparts;        // [B, dslices]
   TileRec *tiles;          // [B, ntiles]
+  uint32_t *tcache;        // [kTabCacheSlots, 2 * kExpTabSize] exp tables by row maximum (bf16 logits)
   AccCounters *ctr;
   const int64_t *request_ids;
   const int32_t *draft_lens;

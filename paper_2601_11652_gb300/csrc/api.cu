@@ -190,6 +190,7 @@ Layout make_layout(const wisp_attn_args *a, const wisp_accept_args *c, int sms, 
     L.req_state = take(sizeof(int32_t) * 5 * (size_t)c->B);
     L.dparts = take(sizeof(DrawPart) * (size_t)c->B * sh.dslices);
     L.tiles = take(sizeof(TileRec) * ((size_t)c->B * sh.ntiles + 1));
+    L.tcache = c->logits_dtype == WISP_BF16 ? take((size_t)kTabCacheSlots * kExpTabBytes) : 0;
     // the greedy variant's argmax partials (8 bytes per row and warp slice) share the statistics'
     // space when they fit, else get their own
     int S = 1, vps = 0;
@@ -333,6 +334,7 @@ AcceptParams accept_params(const wisp_accept_args *c, void *ws, const Layout &L,
   ap.queue = rs + 4 * (size_t)c->B;
   ap.dparts = at<DrawPart>(ws, L.dparts);
   ap.ctr = at<AccCounters>(ws, L.acc_ctr);
+  ap.tcache = bf ? at<uint32_t>(ws, L.tcache) : nullptr;
   ap.request_ids = c->request_ids;
   ap.draft_lens = c->draft_lens;
   ap.logits = c->target_logits;

@@ -129,6 +129,10 @@ __device__ void plan_accept(const PlanParams &p, int64_t *s_warp) {
     p.acc_ctr->n_claimed = 0;
     p.acc_ctr->stats_next = 0;
   }
+  for (int j = tid; j < kTabCacheSlots; j += kThreads) {
+    p.acc_ctr->tab_state[j] = 0;
+    p.acc_ctr->tab_m[j] = 0;
+  }
 }
 
 }  // namespace

@@ -33,6 +33,8 @@ constexpr int kItemsPerSM = 2;     // work items per SM when (request, head) pai
 constexpr int kMinChunk = 256;     // never split a sequence below this many tokens
 constexpr int kChunkAlign = 128;   // chunk starts are multiples of the KV tile
 
+constexpr int kTabCacheSlots = 32;  // exp tables of the draw kept in global memory per launch
+
 // Global counters of one acceptance launch (zeroed by the planner).
 struct AccCounters {
   int32_t n_items;       // statistics items (slices x rows of valid requests)
@@ -48,6 +50,10 @@ struct AccCounters {
   int32_t pad2[31];
   int32_t stats_next;    // next statistics item to claim (its own line)
   int32_t pad3[31];
+  // the draw's exp tables shared through global memory, one per row maximum m (bf16 bits):
+  // state 0 free, 1 being written, 2 ready (tab_m holds its m)
+  int32_t tab_state[kTabCacheSlots];
+  uint32_t tab_m[kTabCacheSlots];
 };
 
 // Byte offsets of every region inside the caller's workspace.
@@ -73,6 +79,7 @@ struct Layout {
   size_t req_state = 0;       // int32 [5, B]: lowest rejecting row, claim, L, finished draw slices, queue
   size_t dparts = 0;          // DrawPart [B, dslices]
   size_t tiles = 0;           // TileRec [B, ntiles]
+  size_t tcache = 0;          // uint32 [kTabCacheSlots, 2 * kExpTabSize]: the draw's exp tables
   // greedy variant
   size_t row_parts = 0;       // argmax partials [total_q_rows, slices]
   size_t total = 0;

@@ -191,5 +191,15 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// Acquire load / release store of a global 32-bit word at GPU scope.
+__device__ __forceinline__ int ld_acquire_gpu(const int *p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_gpu(int *p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
 }  // namespace ptx
 }  // namespace wisp
