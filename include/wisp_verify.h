@@ -130,7 +130,10 @@ typedef struct {
  * Supported: 1 <= V <= 2^24.
  * The kernel decides every comparison exactly up to about 1e-13 relative error: it computes
  * the row normaliser in fp32 with a certified error bound and recomputes it in double-float
- * arithmetic whenever a decision lies inside that bound.
+ * arithmetic whenever a decision lies inside that bound; the extra-token draw sums the weights
+ * exp(z - m) of row L as 2^-56 fixed-point integers (exact, order-free sums) and settles the
+ * sign of p - q with the certified normaliser, weighing undecided elements exactly.
+ * One call is one planner launch and one persistent acceptance kernel on `stream`.
  */
 typedef struct {
   int32_t B, V;
@@ -169,10 +172,12 @@ wisp_status wisp_verify_accept_greedy(const wisp_accept_args *acc, void *workspa
                                       void *stream);
 
 /* Enqueue one whole verification step (Sec. 4.5): attention and acceptance.  The two parts
- * read disjoint inputs; draft_lens must describe the same batch in both structs.  Part of the
- * acceptance pass (its row statistics) runs on a stream owned by the library, forked from and
- * joined back into `stream` with events, so work queued on `stream` afterwards sees the whole
- * step finished. */
+ * read disjoint inputs; draft_lens must describe the same batch in both structs.  One planner
+ * serves both; the attention follows it on `stream`, and the acceptance pass runs on a side
+ * stream owned by the library, forked from and joined back into `stream` with events, so work
+ * queued on `stream` afterwards sees the whole step finished.  Each caller stream gets its own
+ * side stream (created on its first step: make that first call before any stream capture), so
+ * steps on different streams, with different workspaces, run independently. */
 wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args *acc, void *workspace,
                              size_t workspace_bytes, void *stream);
 

@@ -13,14 +13,22 @@ namespace {
 
 constexpr int kMaxDevices = 64;
 
+// wisp_verify_step runs the acceptance pass on a side stream forked from and joined back into the
+// caller's stream with two events.  Each caller stream gets its own side stream, so that steps
+// issued on different streams do not wait for each other; past kMaxSides caller streams the slots
+// are shared (correct, only serialised).
+constexpr int kMaxSides = 32;
+struct SideSlot {
+  cudaStream_t caller = nullptr;
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+};
 struct DeviceInfo {
   int sms = 0;
   bool attrs_done = false;
-  // wisp_verify_step runs the acceptance row statistics on `side`, forked from and joined back
-  // into the caller's stream with these events; step_mu keeps the fork / join of two calls apart
-  cudaStream_t side = nullptr;
-  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
-  std::mutex step_mu;
+  SideSlot sides[kMaxSides];
+  int n_sides = 0;
+  std::mutex step_mu;  // the slot table, and the fork / join of one call kept together
 };
 DeviceInfo g_dev[kMaxDevices];
 std::mutex g_mu;
@@ -38,6 +46,21 @@ const Exp2Table g_exp2 = make_exp2_table();
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+// The side stream and events of caller stream `s` (created on its first step; under d.step_mu).
+SideSlot *side_slot(DeviceInfo &d, cudaStream_t s) {
+  for (int i = 0; i < d.n_sides; ++i)
+    if (d.sides[i].caller == s) return &d.sides[i];
+  if (d.n_sides == kMaxSides) return &d.sides[(uintptr_t)s % kMaxSides];
+  SideSlot &n = d.sides[d.n_sides];
+  if (cudaStreamCreateWithFlags(&n.side, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&n.ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&n.ev_join, cudaEventDisableTiming) != cudaSuccess)
+    return nullptr;
+  n.caller = s;
+  ++d.n_sides;
+  return &n;
+}
+
 wisp_status device_setup(int *dev_out, int *sms_out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return WISP_ERR_CUDA;
@@ -49,9 +72,6 @@ wisp_status device_setup(int *dev_out, int *sms_out) {
     cudaError_t e = attn_simt_setup();
     if (e == cudaSuccess) e = attn_tc_setup();
     if (e == cudaSuccess) e = accept_setup();
-    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&d.side, cudaStreamNonBlocking);
-    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&d.ev_fork, cudaEventDisableTiming);
-    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&d.ev_join, cudaEventDisableTiming);
     if (e != cudaSuccess) return WISP_ERR_CUDA;
     d.sms = sms;
     d.attrs_done = true;
@@ -468,16 +488,21 @@ wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args 
   // CTAs take the SMs the attention's CTAs leave as they finish.
   DeviceInfo &d = g_dev[dev];
   std::lock_guard<std::mutex> lk(d.step_mu);
+  SideSlot *sl = side_slot(d, s);
+  if (!sl) return WISP_ERR_CUDA;
   if ((st = launch_plan(attn, acc, ws, L, sms, true, s)) != WISP_OK) return st;
   const AcceptParams ap = accept_params(acc, ws, L, sms);
   const bool bf = acc->logits_dtype == WISP_BF16;
-  bool ok = cudaEventRecord(d.ev_fork, s) == cudaSuccess && cudaStreamWaitEvent(d.side, d.ev_fork, 0) == cudaSuccess;
-  ok = ok && accept_launch(ap, bf, sms, d.side, false) == cudaSuccess;
-  // join what was forked even after a failed launch, so that `s` never runs ahead of `side`
-  const bool joined = cudaEventRecord(d.ev_join, d.side) == cudaSuccess;
+  // the attention is enqueued first, so that its CTAs take the SMs first; the acceptance CTAs fill
+  // the SMs the attention leaves
+  bool ok = cudaEventRecord(sl->ev_fork, s) == cudaSuccess;
   ok = ok && launch_attention(attn, ws, L, s, true) == WISP_OK;
-  const bool waited = joined && cudaStreamWaitEvent(s, d.ev_join, 0) == cudaSuccess;
-  return ok && waited ? WISP_OK : WISP_ERR_CUDA;
+  const bool forked = ok && cudaStreamWaitEvent(sl->side, sl->ev_fork, 0) == cudaSuccess;
+  ok = forked && accept_launch(ap, bf, sms, sl->side, false) == cudaSuccess;
+  // join what was forked even after a failed launch, so that `s` never runs ahead of `side`
+  const bool joined = !forked || (cudaEventRecord(sl->ev_join, sl->side) == cudaSuccess &&
+                                  cudaStreamWaitEvent(s, sl->ev_join, 0) == cudaSuccess);
+  return ok && joined ? WISP_OK : WISP_ERR_CUDA;
 }
 
 wisp_status wisp_verify_get_device_status(const void *ws, int32_t *code, int64_t *request_id) {
