@@ -1,5 +1,6 @@
 // api.cu -- host side of the C ABI (include/wisp_verify.h): argument checks, workspace
 // carving and kernel launches.  No allocation, no synchronisation on these paths.
+#include <algorithm>
 #include <cmath>
 #include <cstring>
 #include <mutex>
@@ -116,10 +117,10 @@ void accept_slices(const wisp_accept_args *c, int sms, int *slices, int *vps) {
 }
 
 // Work shape of the acceptance kernel: statistics slices per row (enough items, about eight per
-// resident CTA, to balance the persistent CTAs; a slice is a whole number of 4-vector chunks per
+// resident CTA, to balance the persistent CTAs; a slice is a whole number of 3-vector chunks per
 // thread), draw tiles (64 vectors: one warp's share of a draw chunk; no tile records when they
-// would exceed tile_budget bytes) and draw slices per row (about eight per resident CTA over the
-// batch, whole chunks of 256 vectors).
+// would exceed tile_budget bytes) and draw slices per row (at least two, and one item per resident
+// CTA over the batch when it is small; whole chunks of 256 vectors).
 constexpr size_t kTileBudget = (size_t)256 << 20;
 constexpr size_t kNoAllocTileBudget = (size_t)4 << 20;
 struct AcceptShape {
@@ -149,7 +150,9 @@ AcceptShape accept_shape(const wisp_accept_args *c, int sms, size_t tile_budget)
   const bool tiles = B * nt * (int64_t)sizeof(TileRec) <= (int64_t)tile_budget;
   sh.tile_vecs = tiles ? 64 : 0;
   sh.ntiles = tiles ? (int)nt : 0;
-  cut(8 * ctas, B, kAcceptThreads, &sh.dslices, &sh.vpd);
+  // draw slices: one wave of items over the CTAs when the batch is small, and never a whole row
+  // in one item (a request's draw then spreads over at least two CTAs)
+  cut(std::max<int64_t>(ctas, 2 * B), B, kAcceptThreads, &sh.dslices, &sh.vpd);
   return sh;
 }
 
