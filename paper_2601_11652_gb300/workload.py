@@ -316,3 +316,18 @@ def make_small_batch(seed: int, *, B=5, Hq=8, Hkv=2, D=128, V=4096, dtype="bf16"
     return make_batch_from_lengths(
         f"small{seed}", draft_lens=k, context_lens=c, Hq=Hq, Hkv=Hkv, D=D, V=V, dtype=dtype,
         sigma=float(sigma_for_alpha(alpha)), key=key, shuffle_blocks=shuffle_blocks, extra_blocks=3)
+
+
+def make_round(key, *, k, Hq, Hkv, D, V, dtype="bf16", alpha=0.7, prefix=0) -> dict:
+    """One verification round of one session, drawn from `key`: the k + 1 query rows, the k + 1 new
+    K/V rows, k + 1 logit rows, k draft tokens with their distributions and uniforms, one sample
+    uniform; with prefix > 0 also `prefix` K/V rows for the session's first context."""
+    b = make_batch_from_lengths(f"round{key}", draft_lens=[k], context_lens=[prefix], Hq=Hq, Hkv=Hkv, D=D, V=V,
+                                dtype=dtype, sigma=float(sigma_for_alpha(alpha)), key=tuple(key))
+    pos = np.arange(prefix + k + 1)
+    pages = b.block_tables[0, pos // BLOCK_SIZE]
+    kr = b.k_cache[pages, :, pos % BLOCK_SIZE, :]   # [prefix + k + 1, Hkv, D] in token order
+    vr = b.v_cache[pages, :, pos % BLOCK_SIZE, :]
+    return {"prefix_k": kr[:prefix], "prefix_v": vr[:prefix], "q": b.q, "k_new": kr[prefix:], "v_new": vr[prefix:],
+            "logits": b.logits, "draft_tokens": b.draft_tokens, "draft_probs": b.draft_probs,
+            "accept_u": b.accept_uniforms, "sample_u": float(b.sample_uniforms[0])}
