@@ -36,8 +36,10 @@
 
 namespace wisp {
 
-// exp(u) for the bf16 values u of the draw's table (double-float), written by accept_setup
-__device__ ff g_exp_u[kExpTabSize];
+// exp(u) for the bf16 values u of the draw's table (the host's double exp), written by
+// accept_setup as a 64-bit mantissa M in [2^63, 2^64) whose low 8 bits (zero in a double's 53-bit
+// significand) hold E + 128: exp(u) = M 2^(E - 63)
+__device__ unsigned long long g_exp_m64[kExpTabSize];
 
 namespace {
 
@@ -537,21 +539,30 @@ __device__ void ensure_table(float m, Sm &sm, Tab tab, uint32_t &ph, const Accep
   } else {
     const int mi = exp_tab_index((mb >> 16) ^ 0x8000u);  // -m (m is a bf16 value)
     if (mi >= 0) {
-      const ff Em = g_exp_u[mi];
-      ff g[PER];  // every load first: one round trip
+      // exp(u - m) = exp(u) exp(-m) = Mu Mm 2^(Eu + Em - 126): the high 64 bits of the 128-bit
+      // product times 2^(Eu + Em - 62), rounded to units of 2^-56 (integer operations only)
+      const unsigned long long gm = g_exp_m64[mi];
+      const unsigned long long Mm = gm & ~0xFFull;
+      const int Em = (int)(gm & 0xFFu) - 128;
+      constexpr int U = 8;  // entries in flight per thread
+      for (int j0 = 0; j0 < PER; j0 += U) {
+        unsigned long long g[U];
 #pragma unroll
-      for (int j = 0; j < PER; ++j) {
-        const int idx = threadIdx.x + j * kConsumers;
-        g[j] = idx < kExpTabSize ? g_exp_u[idx] : ff{0.0f, 0.0f};
-      }
+        for (int j = 0; j < U; ++j) {
+          const int idx = threadIdx.x + (j0 + j) * kConsumers;
+          g[j] = (j0 + j < PER && idx < kExpTabSize) ? g_exp_m64[idx] : 0ull;
+        }
 #pragma unroll
-      for (int j = 0; j < PER; ++j) {
-        const int idx = threadIdx.x + j * kConsumers;
-        if (idx < kExpTabSize) {
-          const bool used = bf16_bits_to_float(exp_tab_bits(idx)) <= m;
-          const unsigned long long fx = used ? ff_to_fix(ff_mul(g[j], Em)) : 0ull;
-          tab.lo[idx] = (uint32_t)fx;
-          tab.hi[idx] = (uint32_t)(fx >> 32);
+        for (int j = 0; j < U; ++j) {
+          const int idx = threadIdx.x + (j0 + j) * kConsumers;
+          if (j0 + j < PER && idx < kExpTabSize) {
+            const int sh = 6 - ((int)(g[j] & 0xFFu) - 128 + Em);  // >= 6 for u <= m
+            const unsigned long long hi = __umul64hi(g[j] & ~0xFFull, Mm);
+            const bool used = bf16_bits_to_float(exp_tab_bits(idx)) <= m && sh < 64;
+            const unsigned long long fx = used ? ((hi >> (sh - 1)) + 1) >> 1 : 0ull;
+            tab.lo[idx] = (uint32_t)fx;
+            tab.hi[idx] = (uint32_t)(fx >> 32);
+          }
         }
       }
     } else {
@@ -1385,9 +1396,9 @@ namespace {
 
 // ---- the producer (warp 8): next item, bulk copies into the ring ---------------------------------
 // Lane 0: the next work item of this CTA.  A finish task of this CTA first (it ends a request),
-// then draw tickets (their rows are still in L2), then the next statistics item in the level-major
-// order (skipping rows past a known rejection and rows of decided requests).  WORK_EXIT once every valid request is decided, every draw ticket taken and
-// this CTA has nothing pending; WORK_WAIT otherwise.
+// then the next statistics item in the level-major order (skipping rows past a known rejection
+// and rows of decided requests), then draw tickets.  WORK_EXIT once every valid request is
+// decided, every draw ticket taken and this CTA has nothing pending; WORK_WAIT otherwise.
 template <typename LT>
 __device__ int pick(const AcceptParams &p, Sm &sm, Item &d, long long &idle_since, int issued, int &pend) {
   constexpr int E = LTraits<LT>::E;
@@ -1418,6 +1429,30 @@ __device__ int pick(const AcceptParams &p, Sm &sm, Item &d, long long &idle_sinc
     d.nchunks = (int)((d.v1 - d.v0 + kDrawChunk - 1) / kDrawChunk);
     idle_since = -1;
     return WORK_FINISH;
+  }
+  // statistics first: every row's decision as early as possible (a draw can wait; the requests
+  // decided last bound the pass)
+  const int n_items = __ldcg(&c->n_items);
+  while (ld_vol(&c->stats_next) < n_items) {
+    const int t = atomicAdd(&c->stats_next, 1);
+    if (t >= n_items) break;
+    const int2 ent = __ldcg(p.row_order + t / p.sslices);
+    const int r = ent.x, i = ent.y;
+    if (i > ld_vol(p.req_rej + r)) continue;  // past a rejection, or the request is decided
+    d.kind = WORK_STATS;
+    d.r = r;
+    d.i = i;
+    d.s = t % p.sslices;
+    d.k = __ldg(p.draft_lens + r);
+    d.Q0 = __ldg(p.q_row_start + r);
+    d.D0 = __ldg(p.draft_start + r);
+    d.R = d.Q0 + i;
+    d.resid = 0;
+    d.v0 = min(nvec, (int64_t)d.s * p.svps);
+    d.v1 = min(nvec, d.v0 + p.svps);
+    d.nchunks = (int)((d.v1 - d.v0 + kStatsChunk - 1) / kStatsChunk);
+    idle_since = -1;
+    return WORK_STATS;
   }
   // draw tickets: one atomic increment of the head takes the next ticket.  A ticket taken past the
   // entries reserved so far (a race with other producers) stays pending while this CTA goes on with
@@ -1459,28 +1494,6 @@ __device__ int pick(const AcceptParams &p, Sm &sm, Item &d, long long &idle_sinc
     d.nchunks = (int)((d.v1 - d.v0 + kDrawChunk - 1) / kDrawChunk);
     idle_since = -1;
     return WORK_DRAW;
-  }
-  const int n_items = __ldcg(&c->n_items);
-  while (ld_vol(&c->stats_next) < n_items) {
-    const int t = atomicAdd(&c->stats_next, 1);
-    if (t >= n_items) break;
-    const int2 ent = __ldcg(p.row_order + t / p.sslices);
-    const int r = ent.x, i = ent.y;
-    if (i > ld_vol(p.req_rej + r)) continue;  // past a rejection, or the request is decided
-    d.kind = WORK_STATS;
-    d.r = r;
-    d.i = i;
-    d.s = t % p.sslices;
-    d.k = __ldg(p.draft_lens + r);
-    d.Q0 = __ldg(p.q_row_start + r);
-    d.D0 = __ldg(p.draft_start + r);
-    d.R = d.Q0 + i;
-    d.resid = 0;
-    d.v0 = min(nvec, (int64_t)d.s * p.svps);
-    d.v1 = min(nvec, d.v0 + p.svps);
-    d.nchunks = (int)((d.v1 - d.v0 + kStatsChunk - 1) / kStatsChunk);
-    idle_since = -1;
-    return WORK_STATS;
   }
   if (ld_vol(&c->n_claimed) >= __ldcg(&c->n_valid)) {
     fence_sc();
@@ -1790,17 +1803,19 @@ cudaError_t launch_t(const AcceptParams &ap, int sms, cudaStream_t s, bool pdl) 
   return cudaLaunchKernelEx(&cfg, accept_kernel<LT>, ap);
 }
 
-// exp(u) for the table's bf16 values, in double (the host's exp) split into two floats.
-void host_exp_table(ff *out) {
+// exp(u) for the table's bf16 values, in double (the host's exp), as mantissa and exponent:
+// v = f 2^e with f in [0.5, 1) gives M = f 2^64 (exact: 53 significant bits) and E = e - 1.
+void host_exp_table(unsigned long long *out) {
   for (int idx = 0; idx < kExpTabSize; ++idx) {
     const uint32_t sign = (uint32_t)idx / (kExpTabBinades * 128), rem = (uint32_t)idx % (kExpTabBinades * 128);
     const uint32_t bits = (sign << 15) | (((rem >> 7) + kExpTabLo) << 7) | (rem & 0x7Fu);
     const uint32_t f32 = bits << 16;
     float u;
     memcpy(&u, &f32, sizeof u);
-    const double v = std::exp((double)u);
-    out[idx].hi = (float)v;
-    out[idx].lo = (float)(v - (double)out[idx].hi);
+    int e2 = 0;
+    const double f = std::frexp(std::exp((double)u), &e2);
+    const unsigned long long M = (unsigned long long)std::ldexp(f, 64);
+    out[idx] = (M & ~0xFFull) | (unsigned long long)(e2 - 1 + 128);
   }
 }
 
@@ -1810,13 +1825,13 @@ cudaError_t accept_setup() {
   cudaError_t e = set_attr<float>();
   if (e == cudaSuccess) e = set_attr<uint16_t>();
   if (e == cudaSuccess) {
-    static ff host[kExpTabSize];
+    static unsigned long long host[kExpTabSize];
     static bool filled = false;
     if (!filled) {
       host_exp_table(host);
       filled = true;
     }
-    e = cudaMemcpyToSymbol(g_exp_u, host, sizeof host);
+    e = cudaMemcpyToSymbol(g_exp_m64, host, sizeof host);
   }
   return e;
 }
