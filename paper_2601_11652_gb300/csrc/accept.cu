@@ -544,7 +544,7 @@ __device__ void ensure_table(float m, Sm &sm, Tab tab, uint32_t &ph, const Accep
       const unsigned long long gm = g_exp_m64[mi];
       const unsigned long long Mm = gm & ~0xFFull;
       const int Em = (int)(gm & 0xFFu) - 128;
-      constexpr int U = 8;  // entries in flight per thread
+      constexpr int U = PER;  // entries in flight per thread: every load first
       for (int j0 = 0; j0 < PER; j0 += U) {
         unsigned long long g[U];
 #pragma unroll
