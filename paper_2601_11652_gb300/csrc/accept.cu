@@ -16,12 +16,13 @@
 // Draw items (request, slice of row L) for the extra token (Eq. 3): the residual
 // max(0, p_L - q_{L+1}) after a rejection, else p_L, by inverse CDF in ascending token order.  The
 // weights exp(z - m) are exact 64-bit fixed-point numbers (a per-CTA table over the bf16 values,
-// computed in double-float), so every sum is exact and independent of its order.  One pass gives,
-// per slice, the sum over all elements (the exact normaliser) and, over the elements with
-// p > q, the sums of exp(z - m) and of q; the residual mass of a slice is then
+// from the double exp), so every sum is exact and independent of its order.  One pass gives, per
+// slice and per 64-vector tile, the sum over all elements (the exact normaliser) and, over the
+// elements with p > q, the sums of exp(z - m) and of q; the residual mass of a slice is then
 // E_P - Z Q_P once Z is known.  Elements whose sign the fp32 normaliser cannot settle are kept
-// aside and weighed exactly.  The CTA that finishes the last slice of a request finds the slice
-// holding the crossing of u * total, rescans it with the exact normaliser and writes the token.
+// aside and weighed exactly.  The bookkeeping warp of the CTA that finishes the last slice of a
+// request finds the slice and the tile holding the crossing of u * total, rescans that tile with
+// exact weights and writes the token.
 //
 // Nothing waits on an unbounded condition: a CTA that finds no work sleeps briefly and gives up
 // after about two seconds (recording WISP_DEV_TIMEOUT); the only other wait is for a queue entry
@@ -393,7 +394,7 @@ namespace {
 // Warps 0..7 consume (compute from shared memory), warp 8 produces (picks the next item and keeps
 // bulk copies of its rows in flight in a ring of stages), warp 9 keeps the books (slice records,
 // atomics, the row decisions, L, the draw's crossing search).
-enum : int { WORK_EXIT = 0, WORK_WAIT = 1, WORK_STATS = 2, WORK_DRAW = 3, WORK_FINISH = 4 };
+enum : int { WORK_EXIT = 0, WORK_WAIT = 1, WORK_STATS = 2, WORK_DRAW = 3 };
 enum : int { ROW_UNCERTAIN = 100 };  // transient: decided by the exact normaliser
 
 constexpr int kConsumers = kAcceptThreads;    // consumer threads
@@ -407,7 +408,6 @@ constexpr int kDrawChunk = kConsumers;        // vectors per draw chunk: z 4 KB 
 constexpr int kDrawTile = kDrawChunk / (kCW / 2);  // vectors per tile: one warp's share of a draw chunk
 constexpr int kQOffset = 4096;                // the q part of a draw chunk within its stage
 constexpr int kItemSlots = 4;
-constexpr int kFinQ = 8;
 constexpr long long kWaitCycles = 4000000000LL;  // about two seconds: a wait that long is a failure
 constexpr size_t kRingBytes = (size_t)kStages * kStageBytes;
 static_assert(kDrawChunk * 16 <= kQOffset && kQOffset + kDrawChunk * 8 * 4 <= kStageBytes, "draw chunk layout");
@@ -420,23 +420,12 @@ struct Item {
   int64_t v0, v1;  // vectors [v0, v1) of the row streamed
   int nchunks;
   RowRec rec;
-  // finish: the vectors holding the crossing ([v0, v1)) and its local threshold
-  double thr, Zu;
-  int take_last;
   // results of the consumers
   SlicePart sp;
   U96 ea, ep;
   ff qp;
   int n_amb;
   AmbElem amb[kAmbPerSlice];
-};
-
-// A draw to finish on this CTA (posted by the keeper, scheduled by the producer).
-struct FinTask {
-  int r, i, k, resid, take_last;
-  int64_t Q0, D0, v0, v1;  // the vectors to search: one tile, or a whole slice
-  RowRec rec;
-  double thr, Zu;
 };
 
 // The draw's per-CTA exp table (dynamic shared memory): the fixed-point value as two 32-bit words,
@@ -456,16 +445,11 @@ struct Sm {
   RowStats wst[kCW];
   U96 red[2][2][kCW];  // [buffer][e_all, e_p][warp]
   ff qred[2][kCW];
-  double dred[kCW];
   unsigned tab_m_bits;
   int tab_valid;
   int tab_mode;
   int amb_n;
   AmbElem amb[kAmbPerSlice];
-  int first, lastpos;
-  // local finish queue (keeper -> producer)
-  FinTask fq[kFinQ];
-  int fq_head, fq_tail;
   int keeper_done;
   int abort_;
 };
@@ -878,116 +862,105 @@ __device__ void c_draw(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint
   }
 }
 
-// Finish item: the tile holding the crossing of u * total (Eq. 3), chunk by chunk; per thread the
-// exact weight of its vector, a consumer-wide scan in token order, and the element within the
-// thread holding the crossing; or, with take_last, the last element with weight.  Writes the outputs.
+// The exp table for row maximum m from the launch's global cache, if a CTA has published it
+// (bit-identical to a table built here); else none (the direct exp is then used).
+__device__ Tab cached_table(const AcceptParams &p, float m) {
+  const unsigned mb = __float_as_uint(m);
+  if (!p.tcache) return Tab{nullptr, nullptr};
+  const int slot = (int)((mb >> 16) & (kTabCacheSlots - 1));
+  if (ptx::ld_acquire_gpu(&p.ctr->tab_state[slot]) != 2 || ld_vol((const int32_t *)&p.ctr->tab_m[slot]) != (int32_t)mb)
+    return Tab{nullptr, nullptr};
+  uint32_t *t = p.tcache + (size_t)slot * 2 * kExpTabSize;
+  return Tab{t, t + kExpTabSize};
+}
+
+// The extra token (Eq. 3) from vectors [v0, v1) of row L, which hold the crossing of thr (the
+// share of u * total left at v0), by the bookkeeping warp right after it has located them: exact
+// weights of 32 vectors at a time, a warp scan in token order, then the element of the crossing
+// within its vector; with take_last, or when rounding leaves no crossing, the last element with
+// weight.  Writes the request's outputs.
 template <typename LT>
-__device__ void c_finish(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint32_t &ph, const AcceptParams &p) {
+__device__ void keeper_finish(const AcceptParams &p, const Sm &sm, int r, int i, bool resid, int64_t Q0, int64_t D0,
+                              float m, double Zu, int64_t v0, int64_t v1, double thr, bool take_last) {
   constexpr int E = LTraits<LT>::E;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const bool residual = it.resid != 0;
+  const int lane = threadIdx.x & 31;
+  const LT *row = static_cast<const LT *>(p.logits) + (Q0 + i) * (int64_t)p.V;
+  const float *qrow = p.draft_probs + (D0 + i) * (int64_t)p.V;
+  const Tab tab = std::is_same<LT, uint16_t>::value ? cached_table(p, m) : Tab{nullptr, nullptr};
   double carry = 0.0;
-  const double thr = it.thr;
-  const bool tl = it.take_last != 0;  // no crossing to look for: the last element with weight
-  bool found = false;
-  int64_t last_vec = -1;              // (thread 0) the last vector with weight
-  for (int j = 0; j < it.nchunks; ++j) {
-    const int stg = c % kStages;
-    if (!wait_bar(&sm.full[stg], (c / kStages) & 1, sm, p)) return;
-    const char *sb = ring + (size_t)stg * kStageBytes;
-    const int64_t cv0 = it.v0 + (int64_t)j * kDrawChunk;
-    const bool have = cv0 + tid < it.v1;
+  int tok = -1;
+  int64_t last_vec = -1;  // the last vector with weight so far
+  for (int64_t base = v0; base < v1 && tok < 0; base += 32) {
+    const int64_t vi = base + lane;
+    const bool have = vi < v1;
     uint4 w = make_uint4(0, 0, 0, 0);
     float q[E];
 #pragma unroll
-    for (int i = 0; i < E; ++i) q[i] = 0.0f;
+    for (int x = 0; x < E; ++x) q[x] = 0.0f;
     if (have) {
-      w = reinterpret_cast<const uint4 *>(sb)[tid];
-      if (residual) {
-        const float4 *qs = reinterpret_cast<const float4 *>(sb + kQOffset) + (size_t)tid * (E / 4);
-#pragma unroll
-        for (int h = 0; h < E / 4; ++h) {
-          const float4 t = qs[h];
-          q[4 * h] = t.x;
-          q[4 * h + 1] = t.y;
-          q[4 * h + 2] = t.z;
-          q[4 * h + 3] = t.w;
-        }
-      }
+      w = load_vec<LT>(row, vi, p.V, p.vec_z != 0);
+      if (resid) load_q<E>(qrow, vi * E, p.V, p.vec_q != 0, q);
     }
-    __syncwarp();
-    if (lane == 0) ptx::mbar_arrive(&sm.empty[stg]);
-    ++c;
-    const double wv = have ? vec_weight<LT>(w, q, residual, it.rec.m, it.Zu, sm, tab) : 0.0;
+    const double wv = have ? vec_weight<LT>(w, q, resid, m, Zu, sm, tab) : 0.0;
     double incl = wv;
     for (int o = 1; o < 32; o <<= 1) {
       const double t = __shfl_up_sync(0xffffffffu, incl, o);
       if (lane >= o) incl += t;
     }
-    if (lane == 31) sm.dred[warp] = incl;
-    if (tid == 0) {
-      sm.first = INT32_MAX;
-      sm.lastpos = -1;
-    }
-    cbar(sm, ph, p);
-    double off = carry;
-    for (int x = 0; x < warp; ++x) off += sm.dred[x];
-    double total = carry;
-    for (int x = 0; x < kCW; ++x) total += sm.dred[x];
-    incl += off;
-    if (!tl && !found && incl > thr) atomicMin(&sm.first, tid);
-    if (wv > 0.0) atomicMax(&sm.lastpos, tid);
-    cbar(sm, ph, p);
-    if (!tl && !found && sm.first != INT32_MAX) {
-      if (tid == sm.first) {
-        // this thread's elements in order, with exact weights
+    incl += carry;
+    const unsigned pos = __ballot_sync(0xffffffffu, have && wv > 0.0);
+    if (pos) last_vec = base + 31 - __clz(pos);
+    const unsigned hit = take_last ? 0u : __ballot_sync(0xffffffffu, have && incl > thr);
+    if (hit) {
+      const int l0 = __ffs(hit) - 1;
+      int t_ = -1;
+      if (lane == l0) {
+        // this lane's elements in order, with exact weights
         unsigned long long fx[E];
-        weights<LT>(w, it.rec.m, sm, tab, fx);
+        weights<LT>(w, m, sm, tab, fx);
+        double wt[E];
+#pragma unroll
+        for (int x = 0; x < E; ++x) wt[x] = vi * E + x < p.V ? weight_d(fx[x], q[x], resid, Zu) : 0.0;
         const double r2 = thr - (incl - wv);
         double acc = 0.0;
-        int tok = -1, lastv = -1;
-        #pragma unroll
-        for (int i = 0; i < E; ++i) {
-          const int64_t v = (cv0 + tid) * E + i;
-          if (v >= p.V) break;
-          const double wt = weight_d(fx[i], q[i], residual, it.Zu);
-          if (wt > 0.0) lastv = (int)v;
-          acc += wt;
-          if (acc > r2) {
-            tok = (int)v;
-            break;
+        int lastv = -1;
+#pragma unroll
+        for (int x = 0; x < E; ++x) {
+          if (t_ < 0) {
+            if (wt[x] > 0.0) lastv = (int)(vi * E + x);
+            acc += wt[x];
+            if (acc > r2) t_ = (int)(vi * E + x);
           }
         }
-        p.accepted_len[it.r] = it.i;
-        p.next_token[it.r] = tok >= 0 ? tok : lastv;
+        if (t_ < 0) t_ = lastv;
       }
-      found = true;
+      tok = __shfl_sync(0xffffffffu, t_, l0);
+      if (tok < 0) tok = -2;  // the crossing vector had no element with weight after all
+      break;
     }
-    if (tid == 0 && sm.lastpos >= 0) last_vec = cv0 + sm.lastpos;
-    carry = total;
-    cbar(sm, ph, p);  // sm.first / sm.lastpos / sm.dred are rewritten by the next chunk
+    carry = __shfl_sync(0xffffffffu, incl, 31);
   }
-  if (!found && tid == 0) {
-    // rounding left no crossing in the tile (or take_last): the last element with weight
-    int tok = -1;
-    if (last_vec >= 0) {
-      const LT *row = static_cast<const LT *>(p.logits) + (it.Q0 + it.i) * (int64_t)p.V;
-      const float *qrow = p.draft_probs + (it.D0 + it.i) * (int64_t)p.V;
+  if (tok < 0) {
+    // no crossing (take_last, or rounding): the last element with weight
+    tok = -1;
+    if (last_vec >= 0 && lane == 0) {
       const uint4 w = load_vec<LT>(row, last_vec, p.V, p.vec_z != 0);
       float q[E];
-      #pragma unroll
-      for (int i = 0; i < E; ++i) q[i] = 0.0f;
-      if (residual) load_q<E>(qrow, last_vec * E, p.V, p.vec_q != 0, q);
+#pragma unroll
+      for (int x = 0; x < E; ++x) q[x] = 0.0f;
+      if (resid) load_q<E>(qrow, last_vec * E, p.V, p.vec_q != 0, q);
       unsigned long long fx[E];
-      weights<LT>(w, it.rec.m, sm, tab, fx);
-      #pragma unroll
-      for (int i = 0; i < E; ++i) {
-        const int64_t v = last_vec * E + i;
-        if (v < p.V && weight_d(fx[i], q[i], residual, it.Zu) > 0.0) tok = (int)v;
+      weights<LT>(w, m, sm, tab, fx);
+#pragma unroll
+      for (int x = 0; x < E; ++x) {
+        const int64_t v = last_vec * E + x;
+        if (v < p.V && weight_d(fx[x], q[x], resid, Zu) > 0.0) tok = (int)v;
       }
     }
-    p.accepted_len[it.r] = it.i;
-    p.next_token[it.r] = tok;
+  }
+  if (lane == 0) {
+    p.accepted_len[r] = i;
+    p.next_token[r] = tok;
   }
 }
 
@@ -1161,7 +1134,6 @@ __device__ void k_stats(const AcceptParams &p, Sm &sm, const Item &it) {
   try_determine(p, r, k, it.Q0);
 }
 
-// Post a finish task to this CTA's producer (bounded wait for room).
 // One of a tile record's integer sums (over the elements with p > q when pos, else all).
 __device__ __forceinline__ U96 tile_u96(const TileRec *t, bool pos) {
   U96 r = u96_zero();
@@ -1170,25 +1142,11 @@ __device__ __forceinline__ U96 tile_u96(const TileRec *t, bool pos) {
   return r;
 }
 
-__device__ bool post_finish(Sm &sm, const FinTask &f, const AcceptParams &p) {
-  const long long t0 = clock64();
-  while (vload(sm.fq_tail) - vload(sm.fq_head) >= kFinQ) {
-    if (vload(sm.abort_) || clock64() - t0 > kWaitCycles) {
-      if (atomicExch(&sm.abort_, 1) == 0) report(p.status, WISP_DEV_TIMEOUT, nullptr, -1);
-      return false;
-    }
-  }
-  const int t = sm.fq_tail;
-  sm.fq[t % kFinQ] = f;
-  __threadfence_block();
-  vstore(sm.fq_tail, t + 1);
-  return true;
-}
 
 // A draw item is complete: its slice record and the request's count.  The warp that completes the
 // request: exact normaliser (the slices' sums of exp(z - m)), residual mass per slice, the slice
-// holding the crossing of u * total (Eq. 3), the tile within it (from the tile records); the token
-// within the tile is found by a finish item on this CTA's consumers.
+// holding the crossing of u * total (Eq. 3), the tile within it (from the tile records), and the
+// token within the tile (keeper_finish).
 template <typename LT>
 __device__ void k_draw(const AcceptParams &p, Sm &sm, const Item &it) {
   constexpr int E = LTraits<LT>::E;
@@ -1276,24 +1234,9 @@ __device__ void k_draw(const AcceptParams &p, Sm &sm, const Item &it) {
     return;
   }
   const int64_t s0 = (int64_t)d * p.vpd, s1 = min(nvec, s0 + p.vpd);
-  FinTask f;
-  f.r = r;
-  f.i = it.i;
-  f.k = it.k;
-  f.resid = resid ? 1 : 0;
-  f.Q0 = it.Q0;
-  f.D0 = it.D0;
-  f.rec = it.rec;
-  f.Zu = Zu;
   if (p.tile_vecs == 0) {
-    // no tile records (they would not fit): the finish item searches the whole slice
-    if (lane == 0) {
-      f.take_last = take_last;
-      f.v0 = s0;
-      f.v1 = s1;
-      f.thr = thr_d;
-      post_finish(sm, f, p);
-    }
+    // no tile records (they would not fit): the whole slice is searched
+    keeper_finish<LT>(p, sm, r, it.i, resid, it.Q0, it.D0, it.rec.m, Zu, s0, s1, thr_d, take_last != 0);
     return;
   }
   // the tile within slice d
@@ -1354,18 +1297,16 @@ __device__ void k_draw(const AcceptParams &p, Sm &sm, const Item &it) {
     tile = lastpos;
     take_last = 1;
   }
-  if (lane == 0) {
-    if (tile < 0) {
+  if (tile < 0) {
+    if (lane == 0) {
       p.accepted_len[r] = it.i;
       p.next_token[r] = -1;
-      return;
     }
-    f.take_last = take_last;
-    f.v0 = tile * p.tile_vecs;
-    f.v1 = min(nvec, f.v0 + p.tile_vecs);
-    f.thr = thr_t;
-    post_finish(sm, f, p);
+    return;
   }
+  const int64_t t0v = tile * p.tile_vecs;
+  keeper_finish<LT>(p, sm, r, it.i, resid, it.Q0, it.D0, it.rec.m, Zu, t0v, min(nvec, t0v + p.tile_vecs), thr_t,
+                    take_last != 0);
 }
 
 template <typename LT>
@@ -1382,7 +1323,7 @@ __device__ void keeper(const AcceptParams &p, Sm &sm) {
     __syncwarp();
     if (lane == 0) {
       __threadfence_block();
-      vstore(sm.keeper_done, n + 1);  // after any finish task this item posted
+      vstore(sm.keeper_done, n + 1);
       ptx::mbar_arrive(&sm.iq_empty[slot]);
     }
     __syncwarp();
@@ -1395,10 +1336,10 @@ namespace {
 
 
 // ---- the producer (warp 8): next item, bulk copies into the ring ---------------------------------
-// Lane 0: the next work item of this CTA.  A finish task of this CTA first (it ends a request),
-// then the next statistics item in the level-major order (skipping rows past a known rejection
-// and rows of decided requests), then draw tickets.  WORK_EXIT once every valid request is
-// decided, every draw ticket taken and this CTA has nothing pending; WORK_WAIT otherwise.
+// Lane 0: the next work item of this CTA: the next statistics item in the level-major order
+// (skipping rows past a known rejection and rows of decided requests), else a draw ticket.
+// WORK_EXIT once every valid request is decided, every draw ticket taken and this CTA's keeper is
+// done with everything issued; WORK_WAIT otherwise.
 template <typename LT>
 __device__ int pick(const AcceptParams &p, Sm &sm, Item &d, long long &idle_since, int issued, int &pend) {
   constexpr int E = LTraits<LT>::E;
@@ -1406,30 +1347,6 @@ __device__ int pick(const AcceptParams &p, Sm &sm, Item &d, long long &idle_sinc
   AccCounters *c = p.ctr;
   const int Sd = p.dslices;
   if (vload(sm.abort_)) return WORK_EXIT;
-  const int fh = vload(sm.fq_head);
-  if (fh != vload(sm.fq_tail)) {
-    __threadfence_block();
-    const FinTask f = sm.fq[fh % kFinQ];
-    vstore(sm.fq_head, fh + 1);
-    d.kind = WORK_FINISH;
-    d.r = f.r;
-    d.i = f.i;
-    d.k = f.k;
-    d.s = 0;
-    d.resid = f.resid;
-    d.Q0 = f.Q0;
-    d.D0 = f.D0;
-    d.R = f.Q0 + f.i;
-    d.rec = f.rec;
-    d.thr = f.thr;
-    d.Zu = f.Zu;
-    d.take_last = f.take_last;
-    d.v0 = f.v0;
-    d.v1 = f.v1;
-    d.nchunks = (int)((d.v1 - d.v0 + kDrawChunk - 1) / kDrawChunk);
-    idle_since = -1;
-    return WORK_FINISH;
-  }
   // statistics first: every row's decision as early as possible (a draw can wait; the requests
   // decided last bound the pass)
   const int n_items = __ldcg(&c->n_items);
@@ -1499,9 +1416,7 @@ __device__ int pick(const AcceptParams &p, Sm &sm, Item &d, long long &idle_sinc
     fence_sc();
     const int res = ld_vol(&c->q_reserve) * Sd;
     if (pend >= res) pend = -1;  // no entry will ever hold this ticket
-    if (pend < 0 && vload(sm.keeper_done) == issued && ld_vol(&c->q_head) >= res &&
-        vload(sm.fq_head) == vload(sm.fq_tail))
-      return WORK_EXIT;
+    if (pend < 0 && vload(sm.keeper_done) == issued && ld_vol(&c->q_head) >= res) return WORK_EXIT;
   }
   const long long now = clock64();
   if (idle_since < 0) idle_since = now;
@@ -1614,7 +1529,6 @@ __device__ void consumers(const AcceptParams &p, Sm &sm, const char *ring, Tab t
     }
     if (kind == WORK_STATS) c_stats<LT>(sm, it, ring, c, ph, p);
     if (kind == WORK_DRAW) c_draw<LT>(sm, it, bf ? tab : Tab{nullptr, nullptr}, ring, c, ph, p);
-    if (kind == WORK_FINISH) c_finish<LT>(sm, it, bf ? tab : Tab{nullptr, nullptr}, ring, c, ph, p);
     cbar(sm, ph, p);  // every consumer is done with the item
     if (threadIdx.x == 0) ptx::mbar_arrive(&sm.res_ready[slot]);
     if (kind == WORK_EXIT || vload(sm.abort_)) return;
@@ -1651,7 +1565,6 @@ __global__ void __launch_bounds__(kCtaThreads, kAcceptCtasPerSM) accept_kernel(c
     ptx::mbar_init(&sm.cons_bar, kConsumers);
     ptx::fence_mbar_init();
     sm.tab_valid = 0;
-    sm.fq_head = sm.fq_tail = 0;
     sm.keeper_done = 0;
     sm.abort_ = 0;
   }
