@@ -977,13 +977,8 @@ struct DecIn {
 // merged statistics: ROW_ACCEPT / ROW_REJECT when u lies outside the certified interval of the
 // fp32 ratio p(y) / q(y), ROW_UNCERTAIN otherwise (decided with the exact normaliser).
 template <typename LT>
-__device__ int decide(const AcceptParams &p, const RowRec &rec, int64_t R, int64_t D0, int i, DecIn &d) {
-  const int32_t y = __ldg(p.draft_tokens + D0 + i);
+__device__ int decide(const AcceptParams &p, const RowRec &rec, int32_t y, const DecIn &d) {
   if (y < 0 || y >= p.V) return ROW_BAD_TOKEN;
-  const LT *row = static_cast<const LT *>(p.logits) + R * (int64_t)p.V;
-  d.zy = load_scalar(row, y);
-  d.qy = __ldg(p.draft_probs + (D0 + i) * (int64_t)p.V + y);
-  d.u = __ldg(p.accept_u + D0 + i);
   const float zy = d.zy, qy = d.qy, u = d.u;
   if (!(qy >= 0.0f)) return ROW_BAD_PROB;
   if (qy == 0.0f) return ROW_ACCEPT;                                   // a = 1
@@ -1071,25 +1066,47 @@ __device__ double warp_range_weight(const AcceptParams &p, const Sm &sm, const L
 template <typename LT>
 __device__ void k_stats(const AcceptParams &p, Sm &sm, const Item &it) {
   const int lane = threadIdx.x & 31;
-  int last = 0;
-  if (lane == 0) {
-    p.sparts[it.R * p.sslices + it.s] = it.sp;
-    __threadfence();
-    last = atomicAdd(&p.row_cnt[it.R], 1) == p.sslices - 1;
-  }
-  if (!__shfl_sync(0xffffffffu, last, 0)) return;
-  __threadfence();
   const int r = it.r, i = it.i, k = it.k;
+  const LT *lrow = static_cast<const LT *>(p.logits) + it.R * (int64_t)p.V;
+  // the decision's inputs first: the draft token and the uniform, then z(y) and q(y), whose loads
+  // overlap the slice bookkeeping and the merge
+  const bool dec = i < k;
+  const int32_t y = dec ? __ldg(p.draft_tokens + it.D0 + i) : 0;
+  DecIn d{0.0f, 0.0f, dec ? __ldg(p.accept_u + it.D0 + i) : 0.0f};
   RowStats q;
   stats_init(q);
-  if (lane < p.sslices) {
-    const SlicePart *sp = p.sparts + it.R * p.sslices + lane;
-    q.m = __ldcg(&sp->m);
-    q.s.hi = __ldcg(&sp->s_hi);
-    q.s.lo = __ldcg(&sp->s_lo);
-    q.A = __ldcg(&sp->A);
-    q.mfirst = __ldcg(&sp->mfirst);
-    q.nres = __ldcg(&sp->nres);
+  if (p.sslices == 1) {
+    // the item is the whole row: its statistics are the row's
+    if (lane == 0) {
+      q.m = it.sp.m;
+      q.s.hi = it.sp.s_hi;
+      q.s.lo = it.sp.s_lo;
+      q.A = it.sp.A;
+      q.mfirst = it.sp.mfirst;
+      q.nres = it.sp.nres;
+    }
+  } else {
+    int last = 0;
+    if (lane == 0) {
+      p.sparts[it.R * p.sslices + it.s] = it.sp;
+      __threadfence();
+      last = atomicAdd(&p.row_cnt[it.R], 1) == p.sslices - 1;
+    }
+    if (!__shfl_sync(0xffffffffu, last, 0)) return;
+    __threadfence();
+    if (lane < p.sslices) {
+      const SlicePart *sp = p.sparts + it.R * p.sslices + lane;
+      q.m = __ldcg(&sp->m);
+      q.s.hi = __ldcg(&sp->s_hi);
+      q.s.lo = __ldcg(&sp->s_lo);
+      q.A = __ldcg(&sp->A);
+      q.mfirst = __ldcg(&sp->mfirst);
+      q.nres = __ldcg(&sp->nres);
+    }
+  }
+  if (dec && y >= 0 && y < p.V) {
+    d.zy = load_scalar(lrow, y);
+    d.qy = __ldg(p.draft_probs + (it.D0 + i) * (int64_t)p.V + y);
   }
   const RowStats rs = warp_merge(q);
   RowRec rec;
@@ -1098,9 +1115,8 @@ __device__ void k_stats(const AcceptParams &p, Sm &sm, const Item &it) {
   rec.z_lo = rs.s.lo;
   const bool ok = rs.m > -INFINITY && rs.m < INFINITY && rs.s.hi > 0.0f && rs.s.hi < INFINITY && rs.A >= 0.0f;
   rec.dz = ok ? z_bound(rs) : 0.0f;
-  DecIn d{0.0f, 0.0f, 0.0f};
   int code = 0;
-  if (lane == 0) code = !ok ? ROW_BAD_PROB : i == k ? ROW_BONUS : decide<LT>(p, rec, it.R, it.D0, i, d);
+  if (lane == 0) code = !ok ? ROW_BAD_PROB : i == k ? ROW_BONUS : decide<LT>(p, rec, y, d);
   code = __shfl_sync(0xffffffffu, code, 0);
   // the whole draft is validated when row 0 (which the rule always reads) is finished
   if (i == 0 && k > 0) {
@@ -1112,12 +1128,8 @@ __device__ void k_stats(const AcceptParams &p, Sm &sm, const Item &it) {
     if (__any_sync(0xffffffffu, bad)) code = ROW_BAD_TOKEN;
   }
   if (code == ROW_UNCERTAIN) {
-    const LT *row = static_cast<const LT *>(p.logits) + it.R * (int64_t)p.V;
     const int64_t nvec = (p.V + LTraits<LT>::E - 1) / LTraits<LT>::E;
-    const double Zu = warp_range_weight<LT>(p, sm, row, nullptr, rec.m, 0.0, 0, nvec);
-    d.zy = __shfl_sync(0xffffffffu, d.zy, 0);
-    d.qy = __shfl_sync(0xffffffffu, d.qy, 0);
-    d.u = __shfl_sync(0xffffffffu, d.u, 0);
+    const double Zu = warp_range_weight<LT>(p, sm, lrow, nullptr, rec.m, 0.0, 0, nvec);
     // p(y) / q(y) in double precision: z(y) - m is exact, and neither p(y) nor a subnormal q(y)
     // leaves the double range
     const double ratio = exp((double)d.zy - (double)rec.m) * 0x1p56 / (Zu * (double)d.qy);

@@ -45,6 +45,8 @@ SMALL_CASES = [
     # 8 query heads per KV head and k up to 15: up to 128 rows per (request, head), cut into two
     # row groups of at most 64 by the planner, with split chunks
     (6, "bf16", 32, 4, 128, 2000, (8, 15), (0, 2500)),
+    # two row groups at head dim 64 (16 query heads per KV head: 96-128 rows per (request, head))
+    (9, "bf16", 32, 2, 64, 2000, (5, 7), (0, 1500)),
     # head dim 64 with 33-64 rows per (request, head): the second group of softmax warps at D = 64
     (7, "bf16", 16, 2, 64, 3000, (4, 7), (0, 2000)),
     # fp32 inputs (CUDA-core kernel) with up to 128 rows per (request, head)
