@@ -116,11 +116,11 @@ void accept_slices(const wisp_accept_args *c, int sms, int *slices, int *vps) {
   *slices = (int)((nvec + v - 1) / v);
 }
 
-// Work shape of the acceptance kernel: statistics slices per row (enough items, about eight per
-// resident CTA, to balance the persistent CTAs; a slice is a whole number of 3-vector chunks per
-// thread), draw tiles (64 vectors: one warp's share of a draw chunk; no tile records when they
-// would exceed tile_budget bytes) and draw slices per row (at least two, and one item per resident
-// CTA over the batch when it is small; whole chunks of 256 vectors).
+// Work shape of the acceptance kernel: statistics slices per row (about two items per resident
+// CTA over the batch's rows: more, smaller items cost more in per-item set-up and bookkeeping than
+// they gain in balance; a slice is a whole number of 3-vector chunks per thread), draw tiles (64 vectors: one warp's share of a draw chunk; no tile records when they
+// would exceed tile_budget bytes) and draw slices per row (one item per resident CTA over the batch
+// when it is small, up to two per CTA as it grows; whole chunks of 256 vectors).
 constexpr size_t kTileBudget = (size_t)256 << 20;
 constexpr size_t kNoAllocTileBudget = (size_t)4 << 20;
 struct AcceptShape {
@@ -143,16 +143,16 @@ AcceptShape accept_shape(const wisp_accept_args *c, int sms, size_t tile_budget)
     *n = (int)((nvec + v - 1) / v);
   };
   AcceptShape sh;
-  cut(8 * ctas, c->total_q_rows > 0 ? c->total_q_rows : 1, (int64_t)kAcceptThreads * kStatsChunkVecs, &sh.sslices,
+  cut(2 * ctas, c->total_q_rows > 0 ? c->total_q_rows : 1, (int64_t)kAcceptThreads * kStatsChunkVecs, &sh.sslices,
       &sh.svps);
   // a tile is one warp's 64 vectors of a draw chunk; without room for the records, none
   const int64_t nt = (nvec + 63) / 64;
   const bool tiles = B * nt * (int64_t)sizeof(TileRec) <= (int64_t)tile_budget;
   sh.tile_vecs = tiles ? 64 : 0;
   sh.ntiles = tiles ? (int)nt : 0;
-  // draw slices: one wave of items over the CTAs when the batch is small, and never a whole row
-  // in one item (a request's draw then spreads over at least two CTAs)
-  cut(std::max<int64_t>(ctas, 2 * B), B, kAcceptThreads, &sh.dslices, &sh.vpd);
+  // draw slices: one wave of items over the CTAs when the batch is small, up to two waves (and
+  // about three slices per row) as it grows, never a whole row in one item
+  cut(std::max<int64_t>(ctas, std::min<int64_t>(2 * ctas, 3 * B)), B, kAcceptThreads, &sh.dslices, &sh.vpd);
   return sh;
 }
 
