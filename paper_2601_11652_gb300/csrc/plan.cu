@@ -210,15 +210,25 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
   chunk = max64(chunk, kMinChunk);
   chunk = (chunk + kChunkAlign - 1) / kChunkAlign * kChunkAlign;
 
-  // pass 3: items and partial slots (request-major, then KV head, then row group, then chunk)
+  // pass 3: items and partial slots (request-major, then KV head, then row group, then chunk).
+  // Per chunk of kThreads requests: one thread per request sizes its items (block scans), then the
+  // chunk's items are written by consecutive threads (item i by thread i mod kThreads, its request
+  // found by binary search over the chunk's first items), so that the stores coalesce.
+  __shared__ int32_t s_first[kThreads + 1];  // the chunk's requests' first items, relative
+  // per request of the chunk: query rows, chunks (0: no items), first partial, context, first
+  // query row, keys
+  __shared__ int32_t s_rows[kThreads], s_ch[kThreads], s_pf[kThreads], s_ctx[kThreads], s_q0[kThreads], s_nn[kThreads];
   int64_t item_carry = 0, poff_carry = 0;
   for (int base = 0; base < p.B; base += kThreads) {
     const int r = base + tid;
     int64_t n = 0, chunks = 0, rows = 0, nrg = 1, rows0 = 0;
+    int32_t ctx_r = 0;
     if (r < p.B && p.req_flag[r] == REQ_OK) {
-      n = (int64_t)p.context_lens[r] + p.draft_lens[r] + 1;
+      const int32_t k_r = p.draft_lens[r];
+      ctx_r = p.context_lens[r];
+      n = (int64_t)ctx_r + k_r + 1;
       chunks = (n + chunk - 1) / chunk;
-      rows = (int64_t)g * (p.draft_lens[r] + 1);
+      rows = (int64_t)g * (k_r + 1);
       nrg = rows > p.max_rows_item ? 2 : 1;
       rows0 = (rows + nrg - 1) / nrg;  // rows <= 2 * max_rows_item: both groups fit
     }
@@ -230,42 +240,70 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     int64_t ti, tp;
     const int64_t ii = block_scan(nitems, s_warp, &ti);
     const int64_t ip = block_scan(pfl, s_warp, &tp);
+    bool fits = false;
     if (r < p.B) {
       const int64_t first = item_carry + ii - nitems;
       const int64_t pfirst = poff_carry + ip - pfl;
-      const bool fits = first + nitems <= p.max_items && pfirst + pfl <= p.partial_cap;
+      fits = first + nitems <= p.max_items && pfirst + pfl <= p.partial_cap;
       if (!fits && nitems > 0) {
         // cannot happen with the host's bounds; refuse the request rather than overflow
         p.req_flag[r] = REQ_BAD;
         report(p.status, WISP_DEV_UNSUPPORTED, p.request_ids, r);
       }
       p.req_item_begin[r] = (int32_t)first;
-      for (int h = 0; h < 2 * p.Hkv; ++h) p.pair_done[(int64_t)r * p.Hkv * 2 + h] = 0;
       p.req_chunks[r] = fits ? (int32_t)chunks : 0;
-      if (fits) {
-        for (int64_t h = 0; h < p.Hkv; ++h) {
-          for (int64_t rg = 0; rg < nrg; ++rg) {
-            for (int64_t c = 0; c < chunks; ++c) {
-              WorkItem it;
-              it.r = r;
-              it.h = (int32_t)h;
-              it.t0 = (int32_t)(c * chunk);
-              it.t1 = (int32_t)min64(n, (c + 1) * chunk);
-              it.row0 = rg ? (int32_t)rows0 : 0;
-              it.rows = (int32_t)(rg ? rows - rows0 : rows0);
-              it.rg = (int32_t)rg;
-              it.nrg = (int32_t)nrg;
-              it.poff = chunks > 1 ? (int32_t)(pfirst + (h * chunks + c) * (slot_a + slot_b) + (rg ? slot_a : 0)) : -1;
-              it.q0 = p.q_row_start[r];
-              it.ctx = p.context_lens[r];
-              p.items[first + (h * nrg + rg) * chunks + c] = it;
-            }
-          }
-        }
+    }
+    // the chunk's requests in shared memory: first item (relative), rows, chunks (0: no items)
+    s_first[tid] = (int32_t)(ii - nitems);
+    if (tid == kThreads - 1) s_first[kThreads] = (int32_t)ti;
+    s_rows[tid] = (int32_t)rows;
+    s_ch[tid] = fits ? (int32_t)chunks : 0;
+    s_pf[tid] = (int32_t)min64(poff_carry + ip - pfl, INT32_MAX);
+    s_ctx[tid] = ctx_r;
+    s_q0[tid] = r < p.B ? p.q_row_start[r] : 0;
+    s_nn[tid] = (int32_t)n;
+    // per (request, head, row group) finished-chunk counters of the chunk's requests: zeroed, coalesced
+    const int64_t pd0 = (int64_t)base * p.Hkv * 2;
+    const int64_t pd1 = (int64_t)min(p.B, base + kThreads) * p.Hkv * 2;
+    for (int64_t x = pd0 + tid; x < pd1; x += kThreads) p.pair_done[x] = 0;
+    __syncthreads();
+    for (int64_t i = tid; i < ti; i += kThreads) {
+      // the request of item i: the last one whose first item is <= i
+      int lo = 0, hi = kThreads - 1;
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (s_first[mid] <= i) lo = mid;
+        else hi = mid - 1;
       }
+      const int rr = base + lo;
+      const int ch = s_ch[lo];
+      if (ch == 0 || rr >= p.B) continue;  // a refused request (its scan slot is empty)
+      const int rws = s_rows[lo];
+      const int ng = rws > p.max_rows_item ? 2 : 1;
+      const int r0 = (rws + ng - 1) / ng;
+      const int j = (int)(i - s_first[lo]);  // (head, row group, chunk) in that order
+      const int hg = j / ch, c = j - hg * ch;
+      const int h = ng == 2 ? hg >> 1 : hg, rg = ng == 2 ? hg & 1 : 0;
+      const int sa = (r0 * (p.D + 2) + 3) / 4 * 4;
+      const int sb = ng == 2 ? ((rws - r0) * (p.D + 2) + 3) / 4 * 4 : 0;
+      WorkItem it;
+      it.r = rr;
+      it.h = h;
+      it.t0 = (int32_t)(c * chunk);
+      it.t1 = (int32_t)min64(s_nn[lo], (c + 1) * chunk);
+      it.row0 = rg ? r0 : 0;
+      it.rows = rg ? rws - r0 : r0;
+      it.rg = rg;
+      it.nrg = ng;
+      it.poff = ch > 1 ? (int32_t)(s_pf[lo] + (int64_t)(h * ch + c) * (sa + sb) + (rg ? sa : 0)) : -1;
+      it.q0 = s_q0[lo];
+      it.ctx = s_ctx[lo];
+      it.pad = 0;
+      p.items[item_carry + i] = it;
     }
     item_carry += ti;
     poff_carry += tp;
+    __syncthreads();  // s_first / s_rq are rewritten by the next chunk
   }
   // pass 4: dispatch order, longest items first (counting sort on the tile count), so that the
   // persistent kernel ends with its shortest items and its CTAs finish close together

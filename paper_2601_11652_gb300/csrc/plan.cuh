@@ -9,7 +9,7 @@ namespace wisp {
 // [row0, row0 + rows) of the (Hq/Hkv) * (k_r + 1) rows of that head (row = j * (Hq/Hkv) + hh for
 // query position j and head hh of the group).  The row set of a (request, head) is cut into
 // nrg groups when it is larger than the kernel's row limit.
-struct WorkItem {
+struct alignas(16) WorkItem {  // 48 bytes: written and read as three 16-byte vectors
   int32_t r, h, t0, t1;
   int32_t poff;   // offset (floats) of this item's split partials, -1 if the item covers the whole sequence
   int32_t rows;   // query rows of the item
@@ -18,7 +18,9 @@ struct WorkItem {
   int32_t row0;   // first query row of the item within its (request, head)
   int32_t rg;     // row group of the item
   int32_t nrg;    // row groups of its (request, head): 1 or 2
+  int32_t pad;
 };
+static_assert(sizeof(WorkItem) == 48, "work item layout");
 
 struct PlanHeader {
   int32_t n_items;
