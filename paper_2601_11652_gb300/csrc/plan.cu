@@ -44,6 +44,43 @@ __device__ int64_t block_scan(int64_t v, int64_t *s_warp, int64_t *total) {
   return res;
 }
 
+// Inclusive block scans of N int64 per thread at once (one set of barriers for all N): v is replaced
+// by its inclusive values, total[] receives the block sums.  s_w holds N x 32 values.
+template <int N>
+__device__ void block_scan_n(int64_t (&v)[N], int64_t (*s_w)[32], int64_t (&total)[N]) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  for (int d = 1; d < 32; d <<= 1) {
+#pragma unroll
+    for (int x = 0; x < N; ++x) {
+      const int64_t o = __shfl_up_sync(0xffffffffu, v[x], d);
+      if (lane >= d) v[x] += o;
+    }
+  }
+  if (lane == 31) {
+#pragma unroll
+    for (int x = 0; x < N; ++x) s_w[x][w] = v[x];
+  }
+  __syncthreads();
+  if (w == 0) {
+#pragma unroll
+    for (int x = 0; x < N; ++x) {
+      int64_t t = s_w[x][lane];
+      for (int d = 1; d < 32; d <<= 1) {
+        const int64_t o = __shfl_up_sync(0xffffffffu, t, d);
+        if (lane >= d) t += o;
+      }
+      s_w[x][lane] = t;
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int x = 0; x < N; ++x) {
+    v[x] += w > 0 ? s_w[x][w - 1] : 0;
+    total[x] = s_w[x][31];
+  }
+  __syncthreads();
+}
+
 // The acceptance pass's dispatch order and state.  Rows are listed level-major: row index 0 of
 // every valid request, then row index 1, ... (the requests of a level in decreasing draft length, so
 // that request r holds the same position pos(r) in every level it reaches).  The decision of row i
@@ -78,31 +115,28 @@ __device__ void plan_accept(const PlanParams &p, int64_t *s_warp) {
   }
   int64_t nvalid;
   (void)block_scan(nv, s_warp, &nvalid);
-  // n_i: suffix sums of the histogram (buckets in decreasing order, in chunks of kThreads)
-  int64_t carry = 0;
-  for (int base = 0; base < KB; base += kThreads) {
-    const int b = KB - 1 - (base + tid);
-    const int64_t c = b >= 0 ? s_n[b] : 0;
+  static_assert(KB + 1 <= 2 * kThreads, "two histogram buckets per thread");
+  // n_i: suffix sums of the histogram (buckets in decreasing order, two per thread)
+  {
+    const int b0 = KB - 1 - 2 * tid, b1 = b0 - 1;
+    const int64_t h0 = b0 >= 0 ? s_n[b0] : 0, h1 = b1 >= 0 ? s_n[b1] : 0;
     int64_t tot;
-    const int64_t incl = block_scan(c, s_warp, &tot);
-    if (b >= 0) s_n[b] = (int32_t)(carry + incl);
-    carry += tot;
-    __syncthreads();
+    const int64_t incl = block_scan(h0 + h1, s_warp, &tot);
+    if (b0 >= 0) s_n[b0] = (int32_t)(incl - h1);
+    if (b1 >= 0) s_n[b1] = (int32_t)incl;
   }
   if (tid == 0) s_n[KB] = 0;
   __syncthreads();
-  // level starts: exclusive prefix sums of n_i
-  carry = 0;
-  for (int base = 0; base <= KB; base += kThreads) {
-    const int b = base + tid;
-    const int64_t c = b <= KB ? s_n[b] : 0;
-    int64_t tot;
-    const int64_t incl = block_scan(c, s_warp, &tot);
-    if (b <= KB) s_ls[b] = (int32_t)(carry + incl - c);
-    carry += tot;
+  // level starts: exclusive prefix sums of n_i (two per thread)
+  int64_t rows_valid;
+  {
+    const int b0 = 2 * tid, b1 = b0 + 1;
+    const int64_t c0 = b0 <= KB ? s_n[b0] : 0, c1 = b1 <= KB ? s_n[b1] : 0;
+    const int64_t incl = block_scan(c0 + c1, s_warp, &rows_valid);
+    if (b0 <= KB) s_ls[b0] = (int32_t)(incl - c0 - c1);
+    if (b1 <= KB) s_ls[b1] = (int32_t)(incl - c1);
   }
   __syncthreads();
-  const int64_t rows_valid = carry;
   // cursors: in every level, the requests with a larger k come first; bucket k starts at n_{k+1}
   int32_t nxt[2];
   for (int j = 0; j < 2; ++j) {
@@ -142,6 +176,7 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
   // start its own set-up now; it reads the plan only after waiting for this grid to complete
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   __shared__ int64_t s_warp[32];
+  __shared__ int64_t s_warp4[4][32];
   const int tid = threadIdx.x;
   const int g = p.Hq > 0 && p.Hkv > 0 ? p.Hq / p.Hkv : 1;
   const int64_t cap_tokens = (int64_t)p.max_blocks_per_seq * p.block_size;
@@ -163,13 +198,9 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
         n = bad ? 0 : c + k + 1;
       }
     }
-    int64_t tq, td, tn;
-    const int64_t iq = block_scan(r < p.B ? k + 1 : 0, s_warp, &tq);
-    const int64_t id = block_scan(r < p.B ? k : 0, s_warp, &td);
-    const int64_t in = block_scan(n, s_warp, &tn);
-    (void)in;
-    int64_t tv;
-    (void)block_scan(n > 0 ? 1 : 0, s_warp, &tv);
+    int64_t sv[4] = {r < p.B ? k + 1 : 0, r < p.B ? k : 0, n, n > 0 ? 1 : 0}, st[4];
+    block_scan_n<4>(sv, s_warp4, st);
+    const int64_t iq = sv[0], id = sv[1], tq = st[0], td = st[1], tn = st[2], tv = st[3];
     if (r < p.B) {
       const int64_t q0 = carry_q + iq - (k + 1), d0 = carry_d + id - k;
       // a request whose rows fall outside the caller's buffers is never touched
@@ -237,9 +268,9 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     const int64_t slot_a = (rows0 * (p.D + 2) + 3) / 4 * 4;
     const int64_t slot_b = nrg == 2 ? ((rows - rows0) * (p.D + 2) + 3) / 4 * 4 : 0;
     const int64_t pfl = chunks > 1 ? chunks * p.Hkv * (slot_a + slot_b) : 0;
-    int64_t ti, tp;
-    const int64_t ii = block_scan(nitems, s_warp, &ti);
-    const int64_t ip = block_scan(pfl, s_warp, &tp);
+    int64_t sv[2] = {nitems, pfl}, st[2];
+    block_scan_n<2>(sv, s_warp4, st);
+    const int64_t ii = sv[0], ip = sv[1], ti = st[0], tp = st[1];
     bool fits = false;
     if (r < p.B) {
       const int64_t first = item_carry + ii - nitems;
