@@ -113,8 +113,14 @@ __device__ void plan_accept(const PlanParams &p, int64_t *s_warp) {
     p.row_cnt[j] = 0;
     p.row_code[j] = 0;
   }
-  int64_t nvalid;
-  (void)block_scan(nv, s_warp, &nvalid);
+  // valid requests: a warp sum per warp, added into a shared counter
+  __shared__ int32_t s_nvalid;
+  if (tid == 0) s_nvalid = 0;
+  __syncthreads();
+  for (int o = 16; o > 0; o >>= 1) nv += __shfl_xor_sync(0xffffffffu, nv, o);
+  if ((tid & 31) == 0 && nv) atomicAdd(&s_nvalid, nv);
+  __syncthreads();
+  const int64_t nvalid = s_nvalid;
   static_assert(KB + 1 <= 2 * kThreads, "two histogram buckets per thread");
   // n_i: suffix sums of the histogram (buckets in decreasing order, two per thread)
   {
@@ -183,16 +189,21 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
 
   // pass 1: offsets (negative lengths count as 0) and validation
   int64_t carry_q = 0, carry_d = 0, carry_n = 0, carry_v = 0;
+  // with at most kThreads requests, pass 3 reuses what this thread read and decided here
+  int32_t my_k = 0, my_ctx = 0, my_q0 = 0;
+  bool my_ok = false;
   for (int base = 0; base < p.B; base += kThreads) {
     const int r = base + tid;
     int64_t k = 0, n = 0;
     int bad = 0;
     if (r < p.B) {
       k = p.draft_lens[r];
+      my_k = (int32_t)k;
       if (k < 0) { bad = WISP_DEV_BAD_LENGTH; k = 0; }
       if (!bad && k > kMaxDraft) bad = WISP_DEV_UNSUPPORTED;
       if (p.with_attention) {
         const int64_t c = p.context_lens[r];
+        my_ctx = (int32_t)c;
         if (!bad && (c < 0 || c + k + 1 > cap_tokens)) bad = WISP_DEV_BAD_LENGTH;
         if (!bad && (int64_t)g * (k + 1) > kMaxRowsPerHead) bad = WISP_DEV_UNSUPPORTED;
         n = bad ? 0 : c + k + 1;
@@ -209,6 +220,8 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
       p.q_row_start[r] = (int32_t)min64(q0, INT32_MAX);
       p.draft_start[r] = (int32_t)min64(d0, INT32_MAX);
       p.req_flag[r] = bad ? REQ_BAD : REQ_OK;
+      my_q0 = (int32_t)min64(q0, INT32_MAX);
+      my_ok = !bad;
       if (bad) report(p.status, bad, p.request_ids, r);
     }
     carry_q += tq;
@@ -254,9 +267,10 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     const int r = base + tid;
     int64_t n = 0, chunks = 0, rows = 0, nrg = 1, rows0 = 0;
     int32_t ctx_r = 0;
-    if (r < p.B && p.req_flag[r] == REQ_OK) {
-      const int32_t k_r = p.draft_lens[r];
-      ctx_r = p.context_lens[r];
+    const bool one = p.B <= kThreads;  // this thread's request of pass 1
+    if (r < p.B && (one ? my_ok : p.req_flag[r] == REQ_OK)) {
+      const int32_t k_r = one ? my_k : p.draft_lens[r];
+      ctx_r = one ? my_ctx : p.context_lens[r];
       n = (int64_t)ctx_r + k_r + 1;
       chunks = (n + chunk - 1) / chunk;
       rows = (int64_t)g * (k_r + 1);
@@ -291,7 +305,7 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     s_ch[tid] = fits ? (int32_t)chunks : 0;
     s_pf[tid] = (int32_t)min64(poff_carry + ip - pfl, INT32_MAX);
     s_ctx[tid] = ctx_r;
-    s_q0[tid] = r < p.B ? p.q_row_start[r] : 0;
+    s_q0[tid] = r < p.B ? (one ? my_q0 : p.q_row_start[r]) : 0;
     s_nn[tid] = (int32_t)n;
     // per (request, head, row group) finished-chunk counters of the chunk's requests: zeroed, coalesced
     const int64_t pd0 = (int64_t)base * p.Hkv * 2;
