@@ -132,6 +132,15 @@ __device__ __forceinline__ uint32_t exp_tab_bits(int idx) {
   const uint32_t sign = (uint32_t)idx / (kExpTabBinades * 128), rem = (uint32_t)idx % (kExpTabBinades * 128);
   return (sign << 15) | (((rem >> 7) + kExpTabLo) << 7) | (rem & 0x7Fu);
 }
+// Entry of the per-CTA table for the bf16 value with bits b: its own for the table's values, else
+// the zero entry after its sign's range; d >= kExpTabHalf tells the second case (-inf, whose weight
+// is zero, or a value that needs the direct exp).
+__device__ __forceinline__ uint32_t exp_tab_entry(uint32_t b, uint32_t &d) {
+  d = (b & 0x7FFFu) - (uint32_t)(kExpTabLo << 7);
+  return min(d, (uint32_t)kExpTabHalf) + (b >> 15) * (uint32_t)(kExpTabHalf + 1);
+}
+// The entry of the value with compact index idx (0 .. kExpTabSize - 1).
+__device__ __forceinline__ int exp_tab_entry_of(int idx) { return idx + (idx >= kExpTabHalf ? 1 : 0); }
 
 // round(2^56 x) for |x| <= 1 from the bits of x (integer operations only: 64-bit conversions run
 // on the slow FP64 pipe); zero below 2^-126.
@@ -493,7 +502,7 @@ __device__ void ensure_table(float m, Sm &sm, Tab tab, uint32_t &ph, const Accep
   const unsigned mb = __float_as_uint(m);
   if (sm.tab_valid && sm.tab_m_bits == mb) return;
   const int slot = (int)((mb >> 16) & (kTabCacheSlots - 1));
-  uint4 *gt = p.tcache ? reinterpret_cast<uint4 *>(p.tcache + (size_t)slot * 2 * kExpTabSize) : nullptr;
+  uint4 *gt = p.tcache ? reinterpret_cast<uint4 *>(p.tcache + (size_t)slot * 2 * kExpTabEntries) : nullptr;
   if (threadIdx.x == 0) {
     int mode = 0;  // 0 build, 1 build and publish, 2 copy the published table
     if (gt) {
@@ -544,8 +553,8 @@ __device__ void ensure_table(float m, Sm &sm, Tab tab, uint32_t &ph, const Accep
             const unsigned long long hi = __umul64hi(g[j] & ~0xFFull, Mm);
             const bool used = bf16_bits_to_float(exp_tab_bits(idx)) <= m && sh < 64;
             const unsigned long long fx = used ? ((hi >> (sh - 1)) + 1) >> 1 : 0ull;
-            tab.lo[idx] = (uint32_t)fx;
-            tab.hi[idx] = (uint32_t)(fx >> 32);
+            tab.lo[exp_tab_entry_of(idx)] = (uint32_t)fx;
+            tab.hi[exp_tab_entry_of(idx)] = (uint32_t)(fx >> 32);
           }
         }
       }
@@ -553,9 +562,14 @@ __device__ void ensure_table(float m, Sm &sm, Tab tab, uint32_t &ph, const Accep
       for (int idx = threadIdx.x; idx < kExpTabSize; idx += kConsumers) {
         const float u = bf16_bits_to_float(exp_tab_bits(idx));
         const unsigned long long fx = u <= m ? exp_fix_direct(u, m, sm.th, sm.tl).fix : 0ull;
-        tab.lo[idx] = (uint32_t)fx;
-        tab.hi[idx] = (uint32_t)(fx >> 32);
+        tab.lo[exp_tab_entry_of(idx)] = (uint32_t)fx;
+        tab.hi[exp_tab_entry_of(idx)] = (uint32_t)(fx >> 32);
       }
+    }
+    for (int x = threadIdx.x; x < kExpTabEntries - kExpTabSize; x += kConsumers) {  // the zero entries
+      const int e = x == 0 ? kExpTabHalf : kExpTabSize + x;
+      tab.lo[e] = 0u;
+      tab.hi[e] = 0u;
     }
     if (mode == 1) {
       cbar(sm, ph, p);  // the whole table is in shared memory
@@ -582,26 +596,34 @@ __device__ void ensure_table(float m, Sm &sm, Tab tab, uint32_t &ph, const Accep
 template <typename LT>
 __device__ __forceinline__ void weights(const uint4 &w, float m, const Sm &sm, Tab tab,
                                         unsigned long long (&fx)[LTraits<LT>::E]);
+__device__ __noinline__ unsigned long long weight_direct1(uint32_t bits, float m, const Sm &sm) {
+  return bits == 0xFF80u ? 0ull : exp_fix_direct(__uint_as_float(bits << 16), m, sm.th, sm.tl).fix;
+}
 template <>
 __device__ __forceinline__ void weights<uint16_t>(const uint4 &w, float m, const Sm &sm, Tab tab,
                                                   unsigned long long (&fx)[8]) {
-  bool slow = false;
-  int idx[8];
+  uint32_t dmax = 0xFFFFFFFFu;
+  if (tab.lo) {
+    dmax = 0;
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const uint32_t u = (i >> 1) == 0 ? w.x : (i >> 1) == 1 ? w.y : (i >> 1) == 2 ? w.z : w.w;
-    const uint32_t bits = (i & 1) ? (u >> 16) : (u & 0xFFFFu);
-    idx[i] = tab.lo ? exp_tab_index(bits) : -1;
-    if (bits == 0xFF80u) idx[i] = -2;  // -inf: a masked token
-    slow |= idx[i] == -1;
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t u = (i >> 1) == 0 ? w.x : (i >> 1) == 1 ? w.y : (i >> 1) == 2 ? w.z : w.w;
+      const uint32_t bits = (i & 1) ? (u >> 16) : (u & 0xFFFFu);
+      uint32_t d;
+      const uint32_t e = exp_tab_entry(bits, d);
+      dmax = max(dmax, d);
+      fx[i] = ((unsigned long long)tab.hi[e] << 32) | tab.lo[e];
+    }
   }
+  if (dmax >= (uint32_t)kExpTabHalf) {
 #pragma unroll
-  for (int i = 0; i < 8; ++i)
-    fx[i] = idx[i] >= 0 ? ((unsigned long long)tab.hi[idx[i]] << 32) | tab.lo[idx[i]] : 0ull;
-  if (slow) {
-    #pragma unroll
-    for (int i = 0; i < 8; ++i)
-      if (idx[i] == -1) fx[i] = exp_fix_direct(vec_elem<uint16_t>(w, i), m, sm.th, sm.tl).fix;
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t u = (i >> 1) == 0 ? w.x : (i >> 1) == 1 ? w.y : (i >> 1) == 2 ? w.z : w.w;
+      const uint32_t bits = (i & 1) ? (u >> 16) : (u & 0xFFFFu);
+      uint32_t d;
+      exp_tab_entry(bits, d);
+      if (!tab.lo || d >= (uint32_t)kExpTabHalf) fx[i] = weight_direct1(bits, m, sm);
+    }
   }
 }
 template <>
@@ -793,8 +815,9 @@ __device__ void c_draw(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint
       for (int i = 0; i < E; ++i) {
         sa += fx[i];
         if (residual) {
+          // p > q for certain (a negative q included: p - q > p; a NaN q never is)
           const float qi = q[h][i], fl = fix_to_float(fx[i]);
-          const bool pos = qi >= 0.0f && fl > qi * zhi;
+          const bool pos = fl > qi * zhi;
           if (pos) sp += fx[i];
           if (i & 1)
             ff_acc(tq2, pos ? qi : 0.0f);
@@ -807,7 +830,7 @@ __device__ void c_draw(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint
         #pragma unroll
         for (int i = 0; i < E; ++i) {
           const float qi = q[h][i], fl = fix_to_float(fx[i]);
-          if (!(qi >= 0.0f && fl > qi * zhi) && fl > qi * zlo) {
+          if (!(fl > qi * zhi) && fl > qi * zlo) {
             const int a = atomicAdd(&sm.amb_n, 1);
             if (a < kAmbPerSlice) {
               sm.amb[a].e = fx[i];
@@ -870,8 +893,8 @@ __device__ Tab cached_table(const AcceptParams &p, float m) {
   const int slot = (int)((mb >> 16) & (kTabCacheSlots - 1));
   if (ptx::ld_acquire_gpu(&p.ctr->tab_state[slot]) != 2 || ld_vol((const int32_t *)&p.ctr->tab_m[slot]) != (int32_t)mb)
     return Tab{nullptr, nullptr};
-  uint32_t *t = p.tcache + (size_t)slot * 2 * kExpTabSize;
-  return Tab{t, t + kExpTabSize};
+  uint32_t *t = p.tcache + (size_t)slot * 2 * kExpTabEntries;
+  return Tab{t, t + kExpTabEntries};
 }
 
 // The extra token (Eq. 3) from vectors [v0, v1) of row L, which hold the crossing of thr (the
@@ -1556,7 +1579,7 @@ __global__ void __launch_bounds__(kCtaThreads, kAcceptCtasPerSM) accept_kernel(c
   __shared__ Sm sm;
   char *ring = reinterpret_cast<char *>(s_dyn);
   const Tab tab{reinterpret_cast<uint32_t *>(s_dyn + kRingBytes),
-                reinterpret_cast<uint32_t *>(s_dyn + kRingBytes + kExpTabSize * sizeof(uint32_t))};
+                reinterpret_cast<uint32_t *>(s_dyn + kRingBytes + kExpTabEntries * sizeof(uint32_t))};
   // launched as a programmatic dependent of the planner: read nothing before it has completed
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int tid = threadIdx.x, warp = tid >> 5;

@@ -13,10 +13,14 @@ constexpr int kMaxSlices = 32;       // warp slices per row of the greedy varian
 
 // Per-CTA table of exp(u - m) for the bf16 values u with 2^-16 <= |u| < 2^6 (exponent fields
 // kExpTabLo .. kExpTabLo + kExpTabBinades - 1, both signs): 64-bit fixed-point values of the draw.
+// kExpTabSize values; in the table each sign's kExpTabHalf values are followed by a zero entry,
+// which every other bf16 value of that sign reads (kExpTabEntries entries, padded to 4).
 constexpr int kExpTabLo = 111;
 constexpr int kExpTabBinades = 22;
-constexpr int kExpTabSize = 2 * kExpTabBinades * 128;
-constexpr size_t kExpTabBytes = kExpTabSize * 2 * sizeof(uint32_t);  // fixed point, two 32-bit words
+constexpr int kExpTabHalf = kExpTabBinades * 128;
+constexpr int kExpTabSize = 2 * kExpTabHalf;
+constexpr int kExpTabEntries = (2 * (kExpTabHalf + 1) + 3) / 4 * 4;
+constexpr size_t kExpTabBytes = kExpTabEntries * 2 * sizeof(uint32_t);  // fixed point, two 32-bit words
 // Fixed-point scale of the draw's weights: exp(z - m) in [0, 1] is held as round(2^56 exp(z - m)),
 // so that a thread sums up to 2^7 of them in 64 bits and every sum is exact and order-free.
 constexpr int kFixShift = 56;
@@ -105,7 +109,7 @@ struct AcceptParams {
   int32_t *queue;          // [B] requests ready to draw (-1: not yet written)
   DrawPart *dparts;        // [B, dslices]
   TileRec *tiles;          // [B, ntiles]
-  uint32_t *tcache;        // [kTabCacheSlots, 2 * kExpTabSize] exp tables by row maximum (bf16 logits)
+  uint32_t *tcache;        // [kTabCacheSlots, 2 * kExpTabEntries] exp tables by row maximum (bf16 logits)
   AccCounters *ctr;
   const int64_t *request_ids;
   const int32_t *draft_lens;

@@ -271,6 +271,8 @@ PlanParams plan_params(const wisp_attn_args *a, const wisp_accept_args *c, void 
   }
   if (c && c->B > 0 && with_accept) {
     pp.with_accept = 1;
+    pp.split_sms = a != nullptr;
+    pp.V = c->V;
     pp.sslices = accept_shape(c, sms, kTileBudget).sslices;  // (the statistics slices do not depend on the budget)
     pp.row_order = at<int2>(ws, L.row_order);
     pp.row_cnt = at<int32_t>(ws, L.row_cnt);

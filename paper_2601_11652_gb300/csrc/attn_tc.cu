@@ -252,6 +252,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   // only once the planner's grid has completed and its writes are visible
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int n_items = p.header->n_items;
+  if ((int)blockIdx.x >= p.header->attn_ctas) {
+    // the planner leaves this SM to the acceptance pass of the same step: nothing was issued yet
+    if (warp == 1) ptx::tmem_dealloc(tmem, kTmemCols);
+    return;
+  }
   const int g = p.Hq / p.Hkv;
 
   if (warp == 0 || warp == 7) {

@@ -361,7 +361,12 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     const int64_t tiles = ((int64_t)w.t1 - w.t0 + kOrderTile - 1) / kOrderTile;
     return kOrderBuckets - 1 - (int)max64(0, min64(tiles, kOrderBuckets - 1));  // bucket 0: the longest
   };
-  for (int64_t i = tid; i < n_items; i += kThreads) atomicAdd(&s_hist[bucket(i)], 1);
+  int64_t my_tiles = 0;  // KV tile passes of the attention (kOrderTile tokens), this thread's items
+  for (int64_t i = tid; i < n_items; i += kThreads) {
+    atomicAdd(&s_hist[bucket(i)], 1);
+    const WorkItem &w = p.items[i];
+    my_tiles += ((int64_t)w.t1 - w.t0 + kOrderTile - 1) / kOrderTile;
+  }
   __syncthreads();
   {
     static_assert(kOrderBuckets == kThreads, "one bucket per thread in the scan");
@@ -373,14 +378,30 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     __syncthreads();
   }
   for (int64_t i = tid; i < n_items; i += kThreads) p.order[atomicAdd(&s_hist[bucket(i)], 1)] = (int32_t)i;
+  int64_t tiles = 0;
+  block_scan(my_tiles, s_warp, &tiles);
 
   if (tid == 0) {
+    // SMs for the attention in a step whose acceptance pass runs beside it.  Both kernels are
+    // persistent and each fills an SM's shared memory, so the acceptance CTAs start on the SMs the
+    // attention leaves.  Measured on GB300 (bf16, D = 128): with few KV tiles per SM (under ~200
+    // of 64 tokens) the attention is latency-bound and about half the SMs stream its keys as fast
+    // as all of them (32 requests with 0.5-4K contexts: step 0.156 -> 0.129 ms with 80 attention
+    // CTAs of 152); with more it is bound by each SM's streaming rate, and only a few SMs (an
+    // eighth) pay off by starting the acceptance early (2-3% at 256-512 requests; a quarter or
+    // more is slower).  When the acceptance has little vocabulary work per KV tile (under 50
+    // elements: a few requests with long contexts) every SM stays with the attention.
+    const int sms = p.target_items / kItemsPerSM;
+    int na = sms;
+    if (p.with_accept && p.split_sms && tiles > 0 && (int64_t)p.B * p.V >= 50 * tiles)
+      na = tiles < (int64_t)200 * sms ? sms / 2 + 4 : sms - sms / 8;
     PlanHeader hd;
     hd.n_items = (int32_t)n_items;
     hd.chunk_len = (int32_t)chunk;
     hd.partial_floats = (int32_t)min64(poff_carry, p.partial_cap);
     hd.next_item = 0;
-    for (int i = 0; i < 4; ++i) hd.pad[i] = 0;
+    hd.attn_ctas = na;
+    for (int i = 0; i < 3; ++i) hd.pad[i] = 0;
     *p.header = hd;
   }
 }

@@ -27,7 +27,8 @@ struct PlanHeader {
   int32_t chunk_len;
   int32_t partial_floats;
   int32_t next_item;   // work counter of the persistent attention kernel (zeroed by the planner)
-  int32_t pad[4];
+  int32_t attn_ctas;   // CTAs of the tensor-core attention that take items (the others exit at once)
+  int32_t pad[3];
 };
 
 constexpr int kItemsPerSM = 2;     // work items per SM when (request, head) pairs are fewer than SMs
@@ -81,7 +82,7 @@ struct Layout {
   size_t req_state = 0;       // int32 [5, B]: lowest rejecting row, claim, L, finished draw slices, queue
   size_t dparts = 0;          // DrawPart [B, dslices]
   size_t tiles = 0;           // TileRec [B, ntiles]
-  size_t tcache = 0;          // uint32 [kTabCacheSlots, 2 * kExpTabSize]: the draw's exp tables
+  size_t tcache = 0;          // uint32 [kTabCacheSlots, 2 * kExpTabEntries]: the draw's exp tables
   // greedy variant
   size_t row_parts = 0;       // argmax partials [total_q_rows, slices]
   size_t total = 0;
@@ -107,6 +108,9 @@ struct PlanParams {
   int32_t *order;
   // acceptance pass: level-major dispatch order of the logit rows and the launch's state
   int with_accept;
+  int split_sms;               // 1: the acceptance pass runs beside the attention (one step); the
+                               // attention may then leave SMs to it from the start
+  int V;                       // vocabulary of the acceptance pass
   int sslices;                 // statistics slices per row
   int2 *row_order;
   int32_t *row_cnt, *row_code;
