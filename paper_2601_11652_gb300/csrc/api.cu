@@ -378,12 +378,18 @@ AcceptParams accept_params(const wisp_accept_args *c, void *ws, const Layout &L,
 }
 
 // with_accept: the planner also lays out the sampling rule's dispatch order and clears its state
+// accept_apart: the acceptance part is left to launch_plan_accept (on another stream).
 wisp_status launch_plan(const wisp_attn_args *a, const wisp_accept_args *c, void *ws, const Layout &L, int sms,
-                        bool with_accept, cudaStream_t s) {
-  if (cudaMemsetAsync(at<DeviceStatus>(ws, L.status), 0, sizeof(DeviceStatus), s) != cudaSuccess)
-    return WISP_ERR_CUDA;
-  const PlanParams pp = plan_params(a, c, ws, L, sms, with_accept);
+                        bool with_accept, cudaStream_t s, bool accept_apart = false) {
+  PlanParams pp = plan_params(a, c, ws, L, sms, with_accept);
+  pp.accept_apart = accept_apart ? 1 : 0;
   plan_kernel<<<1, 1024, 0, s>>>(pp);
+  return cudaGetLastError() == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
+}
+wisp_status launch_plan_accept(const wisp_attn_args *a, const wisp_accept_args *c, void *ws, const Layout &L,
+                               int sms, cudaStream_t s) {
+  const PlanParams pp = plan_params(a, c, ws, L, sms, true);
+  plan_accept_kernel<<<1, 1024, 0, s>>>(pp);
   return cudaGetLastError() == cudaSuccess ? WISP_OK : WISP_ERR_CUDA;
 }
 
@@ -495,15 +501,16 @@ wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args 
   std::lock_guard<std::mutex> lk(d.step_mu);
   SideSlot *sl = side_slot(d, s);
   if (!sl) return WISP_ERR_CUDA;
-  if ((st = launch_plan(attn, acc, ws, L, sms, true, s)) != WISP_OK) return st;
+  if ((st = launch_plan(attn, acc, ws, L, sms, true, s, true)) != WISP_OK) return st;
   const AcceptParams ap = accept_params(acc, ws, L, sms);
   const bool bf = acc->logits_dtype == WISP_BF16;
-  // the attention is enqueued first, so that its CTAs take the SMs first; the acceptance CTAs fill
-  // the SMs the attention leaves
+  // the attention is enqueued first, so that its CTAs take the SMs first; the acceptance part of
+  // the plan and the acceptance CTAs follow on the side stream, on the SMs the attention leaves
   bool ok = cudaEventRecord(sl->ev_fork, s) == cudaSuccess;
   ok = ok && launch_attention(attn, ws, L, s, true) == WISP_OK;
   const bool forked = ok && cudaStreamWaitEvent(sl->side, sl->ev_fork, 0) == cudaSuccess;
-  ok = forked && accept_launch(ap, bf, sms, sl->side, false) == cudaSuccess;
+  ok = forked && launch_plan_accept(attn, acc, ws, L, sms, sl->side) == WISP_OK;
+  ok = ok && accept_launch(ap, bf, sms, sl->side, false) == cudaSuccess;
   // join what was forked even after a failed launch, so that `s` never runs ahead of `side`
   const bool joined = !forked || (cudaEventRecord(sl->ev_join, sl->side) == cudaSuccess &&
                                   cudaStreamWaitEvent(s, sl->ev_join, 0) == cudaSuccess);

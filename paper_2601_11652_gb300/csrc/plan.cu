@@ -184,6 +184,13 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
   __shared__ int64_t s_warp[32];
   __shared__ int64_t s_warp4[4][32];
   const int tid = threadIdx.x;
+  // the launch's status word starts clear (every kernel of the call reports into it)
+  if (tid == 0) {
+    p.status->code = 0;
+    p.status->pad = 0;
+    p.status->request_id = 0;
+  }
+  __syncthreads();
   const int g = p.Hq > 0 && p.Hkv > 0 ? p.Hq / p.Hkv : 1;
   const int64_t cap_tokens = (int64_t)p.max_blocks_per_seq * p.block_size;
 
@@ -237,7 +244,7 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
       atomicCAS(&p.status->code, 0, (int32_t)WISP_DEV_BAD_LENGTH);
     }
   }
-  if (p.with_accept) plan_accept(p, s_warp);
+  if (p.with_accept && !p.accept_apart) plan_accept(p, s_warp);
   if (!p.with_attention) return;
   __syncthreads();
 
@@ -404,6 +411,14 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     for (int i = 0; i < 3; ++i) hd.pad[i] = 0;
     *p.header = hd;
   }
+}
+
+// The acceptance part of the plan on its own (a step: it runs on the acceptance pass's stream, so
+// that the attention, which waits for the whole planner grid, does not wait for it).  Reads what
+// plan_kernel's first pass wrote (flags and offsets).
+__global__ void __launch_bounds__(kThreads) plan_accept_kernel(const PlanParams p) {
+  __shared__ int64_t s_warp[32];
+  plan_accept(p, s_warp);
 }
 
 }  // namespace wisp

@@ -110,6 +110,7 @@ struct PlanParams {
   int with_accept;
   int split_sms;               // 1: the acceptance pass runs beside the attention (one step); the
                                // attention may then leave SMs to it from the start
+  int accept_apart;            // 1: plan_accept_kernel lays out the acceptance part, not plan_kernel
   int V;                       // vocabulary of the acceptance pass
   int sslices;                 // statistics slices per row
   int2 *row_order;
@@ -120,5 +121,6 @@ struct PlanParams {
 };
 
 __global__ void plan_kernel(const PlanParams p);
+__global__ void plan_accept_kernel(const PlanParams p);
 
 }  // namespace wisp
