@@ -99,3 +99,42 @@ def test_draw_with_shifted_logits_matches_the_oracle(shift):
     got = db.results()
     n, _ = compare_accept(b, got["accepted_len"], got["next_token"], ref)
     assert n >= b.B - 2
+
+
+_SPECIAL = np.array([0x0000, 0x8000, 0x0001, 0x8001,   # +-0, +-smallest subnormal
+                     0x3780, 0xB780, 0x377F, 0xB77F,   # +-2^-16 (the exp table's first value) and just below
+                     0x3781, 0xB781, 0x427F, 0xC27F,   # just above; +-(64 - ulp) (its last)
+                     0x4280, 0xC280, 0xFF80],          # +-64 (past the table), -inf (a masked token)
+                    dtype=np.uint16)
+
+
+@pytest.mark.parametrize("mode", ["near_zero", "large"])
+def test_draw_rows_at_the_exp_table_bounds(oracle_mod, mode):
+    """Draw rows (residual and bonus) whose logits sit on and next to the bounds of the draw's exp
+    table: +-0 and subnormals, +-2^-16 and its neighbours, +-(64 - ulp), +-64, -inf.  Values
+    outside the table take the direct exp (or weigh zero for -inf); all must give the oracle's
+    tokens."""
+    from paper_2601_11652_gb300.device_batch import DeviceBatch
+    rng = np.random.default_rng(21 if mode == "near_zero" else 22)
+    b = wl.make_small_batch(14, B=12, Hq=8, Hkv=2, D=128, V=6000, dtype="bf16", k_range=(1, 6), ctx_range=(0, 100))
+    z = wl.bf16_bits_to_f32(b.logits).astype(np.float32)
+    if mode == "near_zero":
+        z = rng.normal(0.0, 1.0, size=z.shape).astype(np.float32)  # row maxima about 3-4: the specials carry mass
+    else:
+        z = rng.normal(62.0, 1.5, size=z.shape).astype(np.float32)  # maxima past 64
+    bits = wl.f32_to_bf16_bits(z)
+    pick = rng.random(bits.shape) < 0.3
+    bits[pick] = rng.choice(_SPECIAL, size=int(pick.sum()))
+    bits[:, 0] = wl.f32_to_bf16_bits(np.float32(4.0 if mode == "near_zero" else 66.0))  # a finite maximum
+    b.logits = bits
+    ref = oracle_mod.accept(b)
+    assert np.any(ref["accepted_len"] < b.draft_lens) and np.any(ref["accepted_len"] == b.draft_lens), \
+        "residual and bonus draws both occur"
+    db = DeviceBatch.from_host(b)
+    db.step()
+    torch.cuda.synchronize()
+    code, rid = db.device_status()
+    assert code == 0, (code, rid)
+    got = db.results()
+    n, _ = compare_accept(b, got["accepted_len"], got["next_token"], ref)
+    assert n >= b.B - 2
