@@ -597,6 +597,27 @@ def interference(reps: int):
                           "short_slowdown": both / solo_b}), flush=True)
 
 
+def entry_only(args):
+    """One entry point alone on one workload: warm-up calls, then timed calls (L2 flushed before
+    each), median printed.  Used for single-kernel ncu captures on a small case."""
+    import torch
+    from paper_2601_11652_gb300 import build, workload as wl
+    from paper_2601_11652_gb300.device_batch import DeviceBatch
+    build.build()
+    db = DeviceBatch.from_host(wl.make_batch(args.workload))
+    fn = getattr(db, args.entry)
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    ms = _time_loop(fn, args.steps, flush, torch)
+    code, rid = db.device_status()
+    print(json.dumps({"entry": args.entry, "workload": args.workload, "calls": args.steps,
+                      "ms_median": float(np.median(ms)), "device_status": [code, rid]}), flush=True)
+    if code != 0:
+        raise SystemExit(f"device status {code} (request {rid})")
+
+
 def main():
     global SUSTAIN_S
     ap = argparse.ArgumentParser()
@@ -615,8 +636,14 @@ def main():
     ap.add_argument("--lt-reps", type=int, default=20)
     ap.add_argument("--interference", action="store_true", help="solo / co-batched step times of a short and a long "
                     "request (Sec. 3) instead of the benchmark line")
+    ap.add_argument("--entry", choices=["attention", "accept"],
+                    help="call only this entry point, --warmup + --steps times on --workload, and print its "
+                    "median time (a short run for single-kernel profiles) instead of the benchmark line")
     args = ap.parse_args()
     SUSTAIN_S = args.sustain_s
+    if args.entry:
+        entry_only(args)
+        return
     if args.interference:
         interference(20)
         return
