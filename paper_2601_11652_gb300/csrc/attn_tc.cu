@@ -73,10 +73,11 @@ struct Cfg {
   static constexpr int P_BYTES = kBT * kNR * 2; // P^T: [128 tokens][64 rows] bf16
   static constexpr int NSK = D == 128 ? 2 : 4;  // K ring stages
   static constexpr int NSV = D == 128 ? 2 : 4;  // V ring stages
+  static constexpr int NQ = 2;                  // Q buffers: item li's rows in buffer li % NQ
   static constexpr int NP = 2;                  // P buffers: P(n) in buffer n % NP
   static constexpr int RING = 4;                // slots of the item ring
   static constexpr int OFF_Q = 0;
-  static constexpr int OFF_K = OFF_Q + 2 * Q_BYTES;
+  static constexpr int OFF_K = OFF_Q + NQ * Q_BYTES;
   static constexpr int OFF_V = OFF_K + NSK * KV_TILE;
   static constexpr int OFF_P = OFF_V + NSV * KV_TILE;
   static constexpr int OFF_BAR = OFF_P + NP * P_BYTES;
@@ -370,8 +371,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       const WorkItem w = p.items[it];
-      const int qb = li & 1;
-      if (!wait_bar(B.q_empty + qb, ((li >> 1) & 1) ^ 1, s_abort)) { ok = false; break; }
+      const int qb = li % C::NQ;
+      if (!wait_bar(B.q_empty + qb, ((li / C::NQ) & 1) ^ 1, s_abort)) { ok = false; break; }
       ++li;
       // the item's query rows -> Q[qb], row rho (query row row0 + rho = j*g + hh) at MMA row rho.
       // Loads are issued QBATCH at a time per lane before any store.  Rows past `rows` up to the
@@ -440,7 +441,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               s_have = true;
               s_t = 0;
               s_nt = (w.t1 - w.t0 + kBT - 1) / kBT;
-              s_qb = li & 1;
+              s_qb = li % C::NQ;
               s_li = li;
               ++li;
             }
@@ -449,7 +450,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (s_have && n_s < n_pv + 4) {
           const int st = (int)(n_s % C::NSK), sb = n_s & 1;
-          if ((s_t > 0 || ptx::mbar_test_wait(B.q_full + s_qb, (s_li >> 1) & 1)) &&
+          if ((s_t > 0 || ptx::mbar_test_wait(B.q_full + s_qb, (s_li / C::NQ) & 1)) &&
               ptx::mbar_test_wait(B.k_full + st, (n_s / C::NSK) & 1) &&
               ptx::mbar_test_wait(B.s_empty + sb, ((n_s >> 1) & 1) ^ 1)) {
             ptx::tc_fence_after();
