@@ -189,6 +189,19 @@ __device__ __forceinline__ void ff_acc(ff &s, float q) {
   s.hi = t;
 }
 
+// Two such sums at once in packed fp32x2 form: (hi.x, lo.x) += q.x and (hi.y, lo.y) += q.y, each
+// lane rounding exactly as ff_acc (a fused multiply-add by -1 is the rounded difference).
+__device__ __forceinline__ void ff_acc2(float2 &hi, float2 &lo, float2 q) {
+  const float2 m1 = make_float2(-1.0f, -1.0f);
+  const float2 t = __fadd2_rn(hi, q);
+  const float2 bp = __ffma2_rn(hi, m1, t);   // t - hi
+  const float2 ap = __ffma2_rn(bp, m1, t);   // t - bp
+  const float2 e1 = __ffma2_rn(ap, m1, hi);  // hi - ap
+  const float2 e2 = __ffma2_rn(bp, m1, q);   // q - bp
+  lo = __fadd2_rn(lo, __fadd2_rn(e1, e2));
+  hi = t;
+}
+
 __device__ __forceinline__ void u96_add(U96 &a, unsigned long long x) {
   const unsigned long long o = a.lo;
   a.lo += x;
@@ -336,6 +349,34 @@ __device__ __forceinline__ void stats_add_chunk(RowStats &st, const uint4 (&w)[N
   stats_rebase(st, cm);
   const float m = st.m;
   const float span = fminf(m - chunk_min<LT, NV>(w), 104.0f);
+  if (std::is_same<LT, uint16_t>::value) {
+    // bf16: the element pairs of each 32-bit word in packed fp32x2 arithmetic (z - m and the
+    // product with log2 e round exactly as the scalar operations); the pairwise sum adds the pairs
+    // of a vector, then the vectors, then the pair's two halves (depth 3 + 2 + 1 for 24 elements)
+    const float2 nm = make_float2(-m, -m), l2 = make_float2(kLog2e, kLog2e);
+    float2 vp[NV];
+#pragma unroll
+    for (int u = 0; u < NV; ++u) {
+      const uint32_t wd[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+      float2 e[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 z = make_float2(__uint_as_float(wd[i] << 16), __uint_as_float(wd[i] & 0xffff0000u));
+        const float2 x = __fmul2_rn(__fadd2_rn(z, nm), l2);
+        e[i] = make_float2(ex2_approx(x.x), ex2_approx(x.y));
+      }
+      vp[u] = __fadd2_rn(__fadd2_rn(e[0], e[1]), __fadd2_rn(e[2], e[3]));
+    }
+#pragma unroll
+    for (int h = 1; h < NV; h <<= 1) {
+#pragma unroll
+      for (int u = 0; u + h < NV; u += 2 * h) vp[u] = __fadd2_rn(vp[u], vp[u + h]);
+    }
+    const float cs = vp[0].x + vp[0].y;
+    st.s = ff_add_f(st.s, cs);
+    st.A = fmaf(cs, span, st.A);
+    return;
+  }
   float vs[NV];
 #pragma unroll
   for (int u = 0; u < NV; ++u) {
@@ -391,7 +432,7 @@ __device__ __forceinline__ RowStats warp_merge(RowStats st) {
 // and every rescale, the pairwise fp32 sums; the double-float additions are covered by 1e-12.
 __device__ __forceinline__ float z_bound(const RowStats &rs) {
   return 1.05f * ((float)(rs.nres + 2) * kEx2RelErr + 3.0f * 0x1p-24f * (rs.m - rs.mfirst) +
-                  3.0f * 0x1p-24f * (rs.A / rs.s.hi) + 6.0f * 0x1p-24f) +
+                  3.0f * 0x1p-24f * (rs.A / rs.s.hi) + 7.0f * 0x1p-24f) +
          1e-12f;
 }
 
@@ -764,6 +805,7 @@ __device__ void c_draw(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint
   // Z lies in [z_hi (1 - dz), z_hi (1 + dz)]; margins of 2^-20 cover the fp32 roundings of the tests
   const float zhi = rec.z_hi * (1.0f + rec.dz + 0x1p-20f);
   const float zlo = rec.z_hi * (1.0f - rec.dz - 0x1p-20f);
+  const float2 zhi2 = make_float2(zhi, zhi), zlo2 = make_float2(zlo, zlo);
   TileRec *trec = p.tiles + (int64_t)it.r * p.ntiles;
   U96 ea = u96_zero(), ep = u96_zero();
   ff qp = {0.0f, 0.0f};
@@ -804,7 +846,8 @@ __device__ void c_draw(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint
     if (lane == 0) ptx::mbar_arrive(&sm.empty[stg]);
     ++c;
     unsigned long long sa = 0, sp = 0;
-    ff tq = {0.0f, 0.0f}, tq2 = {0.0f, 0.0f};
+    // the q sums of the even (x) and odd (y) elements, as double-floats (hi, lo) in packed form
+    float2 tqh = make_float2(0.0f, 0.0f), tql = make_float2(0.0f, 0.0f);
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       if (!have[h]) continue;
@@ -812,18 +855,23 @@ __device__ void c_draw(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint
       weights<LT>(w[h], rec.m, sm, tab, fx);
       bool amb = false;
 #pragma unroll
-      for (int i = 0; i < E; ++i) {
+      for (int i = 0; i < E; i += 2) {
         sa += fx[i];
+        sa += fx[i + 1];
         if (residual) {
-          // p > q for certain (a negative q included: p - q > p; a NaN q never is)
-          const float qi = q[h][i], fl = fix_to_float(fx[i]);
-          const bool pos = fl > qi * zhi;
-          if (pos) sp += fx[i];
-          if (i & 1)
-            ff_acc(tq2, pos ? qi : 0.0f);
-          else
-            ff_acc(tq, pos ? qi : 0.0f);
-          amb |= !pos && fl > qi * zlo;  // neither certainly positive nor certainly without mass
+          // elements i, i + 1 in packed fp32x2 arithmetic (each operation rounds as its scalar
+          // form).  p > q for certain (a negative q included: p - q > p; a NaN q never is)
+          const float2 qq = make_float2(q[h][i], q[h][i + 1]);
+          const float2 hf = make_float2(__uint2float_rn((uint32_t)(fx[i] >> 32)), __uint2float_rn((uint32_t)(fx[i + 1] >> 32)));
+          const float2 lf = make_float2(__uint2float_rn((uint32_t)fx[i]), __uint2float_rn((uint32_t)fx[i + 1]));
+          const float2 fl = __ffma2_rn(hf, make_float2(0x1p-24f, 0x1p-24f), __fmul2_rn(lf, make_float2(0x1p-56f, 0x1p-56f)));
+          const float2 qh = __fmul2_rn(qq, zhi2), ql = __fmul2_rn(qq, zlo2);
+          const bool p0 = fl.x > qh.x, p1 = fl.y > qh.y;
+          if (p0) sp += fx[i];
+          if (p1) sp += fx[i + 1];
+          ff_acc2(tqh, tql, make_float2(p0 ? qq.x : 0.0f, p1 ? qq.y : 0.0f));
+          // neither certainly positive nor certainly without mass
+          amb |= (!p0 && fl.x > ql.x) || (!p1 && fl.y > ql.y);
         }
       }
       if (amb) {
@@ -841,7 +889,7 @@ __device__ void c_draw(Sm &sm, Item &it, Tab tab, const char *ring, int &c, uint
         }
       }
     }
-    if (residual) tq = ff_add_pos(tq, tq2);
+    const ff tq = ff_add_pos(ff{tqh.x, tql.x}, ff{tqh.y, tql.y});
     // the warp's tile: its sums, warp-wide, into the tile records
     // per lane at most 16 weights of at most 2^56 each
     const U96 A_ = warp_sum_u61(sa), P_ = residual ? warp_sum_u61(sp) : u96_zero();
