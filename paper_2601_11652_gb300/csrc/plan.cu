@@ -363,16 +363,38 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
   const int64_t n_items = min64(item_carry, p.max_items);
   for (int b = tid; b < kOrderBuckets; b += kThreads) s_hist[b] = 0;
   __syncthreads();  // also makes pass 3's items visible to every thread of the block
-  auto bucket = [&](int64_t i) -> int {
-    const WorkItem &w = p.items[i];
-    const int64_t tiles = ((int64_t)w.t1 - w.t0 + kOrderTile - 1) / kOrderTile;
+  // an item's KV tiles: with one chunk of requests (B <= kThreads) from pass 3's shared arrays,
+  // which still describe every request (no global read of the items just written), else from the
+  // item itself
+  const bool one_chunk = p.B <= kThreads;
+  auto item_tiles = [&](int64_t i) -> int64_t {
+    int64_t t0, t1;
+    if (one_chunk) {
+      int lo = 0, hi = kThreads - 1;
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (s_first[mid] <= i) lo = mid;
+        else hi = mid - 1;
+      }
+      const int ch = max(1, s_ch[lo]);
+      const int c = (int)(i - s_first[lo]) % ch;  // item = (head, row group) * ch + chunk
+      t0 = (int64_t)c * chunk;
+      t1 = min64(s_nn[lo], t0 + chunk);
+    } else {
+      const WorkItem &w = p.items[i];
+      t0 = w.t0;
+      t1 = w.t1;
+    }
+    return (t1 - t0 + kOrderTile - 1) / kOrderTile;
+  };
+  auto bucket_of = [&](int64_t tiles) -> int {
     return kOrderBuckets - 1 - (int)max64(0, min64(tiles, kOrderBuckets - 1));  // bucket 0: the longest
   };
   int64_t my_tiles = 0;  // KV tile passes of the attention (kOrderTile tokens), this thread's items
   for (int64_t i = tid; i < n_items; i += kThreads) {
-    atomicAdd(&s_hist[bucket(i)], 1);
-    const WorkItem &w = p.items[i];
-    my_tiles += ((int64_t)w.t1 - w.t0 + kOrderTile - 1) / kOrderTile;
+    const int64_t t = item_tiles(i);
+    atomicAdd(&s_hist[bucket_of(t)], 1);
+    my_tiles += t;
   }
   __syncthreads();
   {
@@ -384,7 +406,7 @@ __global__ void __launch_bounds__(kThreads) plan_kernel(const PlanParams p) {
     s_hist[tid] = excl;
     __syncthreads();
   }
-  for (int64_t i = tid; i < n_items; i += kThreads) p.order[atomicAdd(&s_hist[bucket(i)], 1)] = (int32_t)i;
+  for (int64_t i = tid; i < n_items; i += kThreads) p.order[atomicAdd(&s_hist[bucket_of(item_tiles(i))], 1)] = (int32_t)i;
   int64_t tiles = 0;
   block_scan(my_tiles, s_warp, &tiles);
 
