@@ -151,8 +151,10 @@ AcceptShape accept_shape(const wisp_accept_args *c, int sms, size_t tile_budget)
   sh.tile_vecs = tiles ? 64 : 0;
   sh.ntiles = tiles ? (int)nt : 0;
   // draw slices: one wave of items over the CTAs when the batch is small, up to two waves (and
-  // about three slices per row) as it grows, never a whole row in one item
-  cut(std::max<int64_t>(ctas, std::min<int64_t>(2 * ctas, 3 * B)), B, kAcceptThreads, &sh.dslices, &sh.vpd);
+  // about three slices per row) as it grows, and at least two per row (a slice keeps at most
+  // kAmbPerSlice undecided elements; past that the bookkeeper weighs the slice exactly alone)
+  cut(std::max<int64_t>(2 * B, std::max<int64_t>(ctas, std::min<int64_t>(2 * ctas, 3 * B))), B, kAcceptThreads,
+      &sh.dslices, &sh.vpd);
   return sh;
 }
 

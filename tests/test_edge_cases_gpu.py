@@ -145,3 +145,11 @@ def test_residual_without_mass_draws_from_p(oracle_mod):
         b.accept_uniforms[ds[r]] = np.float32(0.9)
     got, ref = _check(oracle_mod, b, "accept", with_attention=False)
     assert np.all(ref["accepted_len"] == 0)
+
+
+def test_batch_past_two_draw_waves(oracle_mod):
+    """B = 700 requests (more than twice the 304 acceptance CTAs): statistics items are whole rows
+    and the draw keeps two slices per row; every request matches the oracle."""
+    b = wl.make_small_batch(31, B=700, Hq=8, Hkv=2, D=128, V=6000, dtype="bf16", k_range=(0, 4), ctx_range=(0, 64))
+    got, ref = _check(oracle_mod, b)
+    assert np.any(ref["accepted_len"] < b.draft_lens) and np.any(ref["accepted_len"] == b.draft_lens)
