@@ -1285,28 +1285,34 @@ __device__ void k_draw(const AcceptParams &p, Sm &sm, const Item &it) {
     const double t = warp_range_weight<LT>(p, sm, row, qrow, it.rec.m, Zu, a, b);
     if (lane == d) sd = t;
   }
-  // total in slice order (lane 0)
-  double S = 0.0;
-  for (int d = 0; d < Sd; ++d) S += __shfl_sync(0xffffffffu, sd, d);
+  // the slices' masses in slice order: an inclusive warp scan (lane d: slices 0..d), the total from
+  // the last lane, so that the crossing search below reads the same prefix sums as the total
+  auto slice_scan = [&](double v) {
+    double incl = lane < Sd ? v : 0.0;
+    for (int o = 1; o < 32; o <<= 1) {
+      const double t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    return incl;
+  };
+  double incl = slice_scan(sd);
+  double S = __shfl_sync(0xffffffffu, incl, 31);
   if (resid && !(S > 0.0)) {
     // the residual has no mass (only through rounding): draw from p_L instead
     resid = false;
     sd = se;
-    S = 0.0;
-    for (int d = 0; d < Sd; ++d) S += __shfl_sync(0xffffffffu, sd, d);
+    incl = slice_scan(sd);
+    S = __shfl_sync(0xffffffffu, incl, 31);
   }
   const double thr = (double)__ldg(p.sample_u + r) * S;
-  double run = 0.0, thr_d = 0.0;
-  int owner = -1, lastd = -1;
-  for (int d = 0; d < Sd; ++d) {
-    const double t = __shfl_sync(0xffffffffu, sd, d);
-    if (owner < 0 && run + t > thr) {
-      owner = d;
-      thr_d = thr - run;
-    }
-    run += t;
-    if (t > 0.0) lastd = d;
-  }
+  const unsigned hitd = __ballot_sync(0xffffffffu, lane < Sd && incl > thr);
+  const unsigned massd = __ballot_sync(0xffffffffu, lane < Sd && sd > 0.0);
+  const int owner = hitd ? __ffs(hitd) - 1 : -1;
+  const int lastd = massd ? 31 - __clz(massd) : -1;
+  // the share of thr left at the owner's first element: thr minus the scan's prefix before it
+  const double before = __shfl_sync(0xffffffffu, incl, owner > 0 ? owner - 1 : 0);
+  const double thr_d = owner > 0 ? thr - before : owner == 0 ? thr : 0.0;
+  double run = 0.0;
   int take_last = owner < 0 ? 1 : 0;  // rounding left no crossing: the last token with mass
   const int d = owner >= 0 ? owner : lastd;
   if (d < 0) {  // no token has mass (cannot happen for a valid row)
