@@ -233,7 +233,10 @@ def cpu_baseline(batch, budget_s=10.0):
 def run_reference(args, batch):
     """The oracle as the reference arm: each step is a bounded sample of the workload."""
     t_one = time_oracle(batch, 0.0)[2]
-    per_step = max(1, int(3.0 / max(t_one, 1e-3)))
+    # about 3 s of oracle work a step, less when many steps are asked for (the whole run stays
+    # within a few minutes); at least one request a step
+    per_step_s = min(3.0, 240.0 / max(1, args.steps + args.warmup))
+    per_step = max(1, int(per_step_s / max(t_one, 1e-3)))
     for i in range(args.warmup):
         time_oracle(batch, 0.0, start=i)
     ms, verified, done, threads = [], 0, 0, 1
