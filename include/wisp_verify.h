@@ -173,11 +173,14 @@ wisp_status wisp_verify_accept_greedy(const wisp_accept_args *acc, void *workspa
 
 /* Enqueue one whole verification step (Sec. 4.5): attention and acceptance.  The two parts
  * read disjoint inputs; draft_lens must describe the same batch in both structs.  One planner
- * serves both; the attention follows it on `stream`, and the acceptance pass runs on a side
- * stream owned by the library, forked from and joined back into `stream` with events, so work
- * queued on `stream` afterwards sees the whole step finished.  Each caller stream gets its own
- * side stream (created on its first step: make that first call before any stream capture), so
- * steps on different streams, with different workspaces, run independently. */
+ * serves both; the attention follows it on `stream`, and the acceptance pass (with the
+ * acceptance part of the plan) runs on a side stream owned by the library, forked from and
+ * joined back into `stream` with events, so work queued on `stream` afterwards sees the whole step
+ * finished.  The planner sizes the attention from the batch: when the attention is small next to
+ * the acceptance work, part of its CTAs exit at once and the acceptance pass starts on their SMs
+ * (results are the same either way).  Each caller stream gets its own side stream (created on its
+ * first step: make that first call before any stream capture), so steps on different streams,
+ * with different workspaces, run independently. */
 wisp_status wisp_verify_step(const wisp_attn_args *attn, const wisp_accept_args *acc, void *workspace,
                              size_t workspace_bytes, void *stream);
 
