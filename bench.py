@@ -609,7 +609,7 @@ def entry_only(args):
     pool = None
     if args.entry == "accept":
         dt = torch.bfloat16 if b.dtype == "bf16" else torch.float32
-        pool = (torch.zeros(16, dtype=dt, device="cuda"), torch.zeros(16, dtype=dt, device="cuda"))
+        pool = tuple(torch.zeros((1, b.Hkv, 16, b.D), dtype=dt, device="cuda") for _ in range(2))
     db = DeviceBatch.from_host(b, pool=pool)
     fn = getattr(db, args.entry)
     for _ in range(args.warmup):
