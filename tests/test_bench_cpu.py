@@ -1,5 +1,6 @@
 """CPU: the host-side arithmetic of bench.py -- algorithmic bytes, the per-kernel source hashes
-that decide whether a committed ncu summary still describes the sources, and the clock summary."""
+that decide whether a committed ncu summary still describes the sources, the clock summary -- and
+the reference arm's JSON line."""
 import os
 import shutil
 
@@ -102,3 +103,22 @@ def test_issue_roofline_from_the_profile(tmp_path, monkeypatch):
     with open(root / "paper_2601_11652_gb300" / "csrc" / "accept.cu", "a") as f:
         f.write("\n")
     assert bench._profile_inst("accept", "demo") is None
+
+
+def test_reference_arm_prints_the_contract_line():
+    """bench.py --impl reference: the oracle timed on the host cores on the workload's requests,
+    one JSON line with the reference keys (here the small fp32 workload, one short step)."""
+    import json
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference", "--workload",
+                          "tiny_f32", "--steps", "1", "--warmup", "0"], capture_output=True, text=True, timeout=300,
+                         cwd=root)
+    assert out.returncode == 0, out.stderr[-2000:]
+    line = json.loads(out.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["steps"] == 1 and line["value"] > 0
+    assert line["unit"] == "verified_tokens/s" and line["higher_is_better"] is True
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
+    assert line["config"]["workload"] == "tiny_f32"
